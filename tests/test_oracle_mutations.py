@@ -1,0 +1,123 @@
+"""Plant plausible mistakes in the oracle (on the CPU) and check that the pins
+in ``test_oracle_pins.py`` catch each one."""
+import numpy as np
+import pytest
+
+import oracle
+import oracle.moe as M
+import tests.test_oracle_pins as P
+
+
+def _patch(monkeypatch, name, fn):
+    """Replace an oracle function both in its module and in the package namespace."""
+    monkeypatch.setattr(M, name, fn)
+    monkeypatch.setattr(oracle, name, fn)
+
+
+def _expect_failure(fn, *args):
+    with pytest.raises(AssertionError):
+        fn(*args)
+
+
+def test_dropped_term_in_swiglu_backward_is_caught(monkeypatch):
+    def bad(dY_e, X_e, g_e, u_e, wg_e, wu_e, w2_e):
+        sg = M.sigmoid(g_e)
+        a_e = g_e * sg * u_e
+        dA = np.matmul(dY_e, w2_e)
+        dg = dA * u_e * sg * (g_e * (1.0 - sg))          # "1 +" dropped
+        du = dA * (g_e * sg)
+        return (np.matmul(dg, wg_e) + np.matmul(du, wu_e), np.matmul(dg.T, X_e),
+                np.matmul(du.T, X_e), np.matmul(dY_e.T, a_e))
+    _patch(monkeypatch, "expert_ffn_bwd_one", bad)
+    _expect_failure(P.test_backward_matches_central_differences, False)
+    _expect_failure(P.test_single_expert_backward_matches_autograd)
+
+
+def test_wrong_sign_in_router_backward_is_caught(monkeypatch):
+    orig = M.route_bwd
+
+    def bad(x, w_router, idx, prob, dprob):
+        dz, dxr, dwr = orig(x, w_router, idx, prob, dprob)
+        return -dz, -dxr, -dwr
+    _patch(monkeypatch, "route_bwd", bad)
+    _expect_failure(P.test_backward_matches_central_differences, False)
+
+
+def test_tie_to_higher_index_is_caught(monkeypatch):
+    orig_sorted = sorted
+
+    def bad_topk(z, K):
+        T, E = z.shape
+        s = M.softmax_rows(z)
+        idx = np.empty((T, K), dtype=np.int64)
+        prob = np.empty((T, K))
+        for t in range(T):
+            chosen = orig_sorted(range(E), key=lambda e: (-z[t, e], -e))[:K]
+            d = sum(s[t, e] for e in chosen)
+            idx[t] = chosen
+            prob[t] = [s[t, e] / d for e in chosen]
+        return idx, prob
+    _patch(monkeypatch, "top_k_route", bad_topk)
+    _expect_failure(P.test_topk_ties_go_to_lower_index)
+
+
+def test_missing_renormalisation_is_caught(monkeypatch):
+    def bad_topk(z, K):
+        T, E = z.shape
+        s = M.softmax_rows(z)
+        idx = np.empty((T, K), dtype=np.int64)
+        prob = np.empty((T, K))
+        for t in range(T):
+            chosen = sorted(range(E), key=lambda e: (-z[t, e], e))[:K]
+            idx[t] = chosen
+            prob[t] = [s[t, e] for e in chosen]
+        return idx, prob
+    _patch(monkeypatch, "top_k_route", bad_topk)
+    _expect_failure(P.test_topk_matches_brute_force_random, 6, 3)
+    _expect_failure(P.test_identical_experts_give_dense_ffn_for_any_routing)
+
+
+def test_transposed_down_projection_is_caught(monkeypatch):
+    def bad(X_e, wg_e, wu_e, w2_e):
+        g = np.matmul(X_e, wg_e.T)
+        u = np.matmul(X_e, wu_e.T)
+        a = M.silu(g) * u
+        return g, u, a, np.matmul(a, w2_e)  # w2 used untransposed
+    _patch(monkeypatch, "expert_ffn_one", bad)
+    # square D = F makes the mistaken product well formed
+    def square_case():
+        p = P._small_layer(T=30, D=6, E=4, K=2, F=6, seed=7)
+        fwd = M.layer_forward(p["x"], p["w_router"], p["w_gate"], p["w_up"], p["w2"], K=2)
+        for e in range(4):
+            lo, hi = fwd["offsets"][e], fwd["offsets"][e + 1]
+            ref = P._dense_swiglu_torch(p["x"][fwd["token_of_row"][lo:hi]], p["w_gate"][e], p["w_up"][e], p["w2"][e])
+            np.testing.assert_allclose(fwd["y_perm"][lo:hi], ref.numpy(), rtol=1e-12, atol=1e-12)
+    _expect_failure(square_case)
+
+
+def test_unstable_permutation_is_caught(monkeypatch):
+    def bad(idx, E):
+        T, K = idx.shape
+        flat = idx.reshape(-1).tolist()
+        order = sorted(range(T * K), key=lambda s: (flat[s], -(s // K)))
+        ros = np.empty(T * K, dtype=np.int64)
+        tor = np.empty(T * K, dtype=np.int64)
+        for r, s in enumerate(order):
+            ros[s] = r
+            tor[r] = s // K
+        off = np.concatenate([[0], np.cumsum(np.bincount(flat, minlength=E))])
+        return off, ros, tor
+    _patch(monkeypatch, "expert_permutation", bad)
+    _expect_failure(P.test_permutation_vs_stable_argsort, 50, 8, 2)
+
+
+def test_wrong_combine_weight_is_caught(monkeypatch):
+    def bad(y_perm, prob_perm, row_of_slot, T, K):
+        y = np.zeros((T, y_perm.shape[1]))
+        for t in range(T):
+            for k in range(K):
+                r = row_of_slot[t * K + k]
+                y[t] += prob_perm[row_of_slot[t * K]] * y_perm[r]   # always slot 0's weight
+        return y
+    _patch(monkeypatch, "combine", bad)
+    _expect_failure(P.test_combine_of_dispatch_with_identity_experts_returns_x)
