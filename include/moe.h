@@ -1,0 +1,213 @@
+/*
+ * moe.h -- C ABI of the GB300 (sm_103a) dropless routed MoE layer library.
+ *
+ * One routed Mixture-of-Experts layer, forward and backward, on one GPU.
+ * The layer is the object of the paper's Eq. 1 (Sec. 1): dropless routing
+ * with no capacity padding, each token dispatched to its K routed experts as a
+ * hidden vector of width D (b_x bytes per element) plus one routed probability
+ * (b_p = 4 bytes, fp32).  Sec. 4.1 (footnote on the all-to-all dispatcher)
+ * names the six transfers of one layer: hidden dispatch, probability dispatch
+ * and hidden combine forward, plus their three inverses backward.  With every
+ * expert on one GPU those transfers become the in-HBM permutes below
+ * (moe_dispatch, moe_combine, moe_combine_bwd, moe_dispatch_bwd).  Sec. 5.2
+ * names the building blocks (grouped-GEMM experts, fused permute); the
+ * LatentMoE projections (Sec. 1 levers list, Table 2) are moe_latent_proj*.
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ *  - T = S * GBS tokens, TK = T * K routed slots; slot s = t * K + k is token
+ *    t's k-th routed expert.  "Rows" are the slots in expert-grouped order:
+ *    expert e owns rows [expert_offsets[e], expert_offsets[e+1]), and within
+ *    an expert rows are ordered by token (a counting sort, stable in t).
+ *  - Every data pointer is a DEVICE pointer owned by the caller, row-major and
+ *    contiguous, 16-byte aligned.  The library never allocates or frees
+ *    caller-visible memory; scratch comes from the caller-provided workspace
+ *    `ws` of `ws_bytes` bytes (size from moe_workspace_size).
+ *  - `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *    stream).  Every call only enqueues work on that stream and returns; there
+ *    is no host synchronisation (moe_check_device_status excepted).
+ *  - Activation and weight storage dtype is shape->x_dtype (MOE_BF16: b_x = 2,
+ *    MOE_F32: b_x = 4).  Probabilities, logits and their gradients are fp32;
+ *    weight gradients are written fp32; routing indices and the permutation
+ *    are int32.  All accumulations are fp32.  MOE_F32 uses plain fp32 FMA
+ *    throughout (no TF32).
+ *  - Return value: MOE_OK (0) or a negative moe_status.  On error nothing has
+ *    been enqueued.  Errors found on the device (an out-of-range expert index,
+ *    a bounded wait that expired) set a device status word that
+ *    moe_check_device_status reads.
+ *
+ * Weight layouts
+ *  - w_router [E, Din]: logits z = x . w_router^T (Din = H for LatentMoE,
+ *    else D).
+ *  - w1 [E, 2F, D]: gate and up projections packed by moe_pack_w1, in blocks
+ *    of 64 rows: rows [128 i, 128 i + 64) are gate rows 64 i .. 64 i + 63 and
+ *    rows [128 i + 64, 128 i + 128) are the up rows of the same 64 features.
+ *    The saved pre-activation h [TK, 2F] and its gradient use the same order.
+ *  - w2 [E, D, F]: Y = a . w2_e^T.
+ *  - Gradients dw1 / dw2 / dw_router have the layouts of w1 / w2 / w_router.
+ */
+#ifndef MOE_GB300_H
+#define MOE_GB300_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    MOE_OK = 0,
+    MOE_ERR_SHAPE = -1,       /* non-positive or inconsistent sizes, K > E, E > 256, D or F not a multiple of 64, overflow */
+    MOE_ERR_DTYPE = -2,       /* unknown x_dtype */
+    MOE_ERR_ALIGN = -3,       /* a pointer not 16-byte aligned */
+    MOE_ERR_NULL = -4,        /* a required pointer is NULL */
+    MOE_ERR_WORKSPACE = -5,   /* ws_bytes smaller than moe_workspace_size() */
+    MOE_ERR_CUDA = -6,        /* a CUDA runtime call or launch failed (see moe_last_cuda_error) */
+    MOE_ERR_DEVICE = -7,      /* the device status word is set (moe_check_device_status) */
+    MOE_ERR_UNSUPPORTED = -8  /* valid request this build does not implement */
+} moe_status;
+
+typedef enum { MOE_BF16 = 0, MOE_F32 = 1 } moe_dtype;
+
+/* Eq. 1 symbols: S sequence length, GBS global batch, K routed top-K, D
+ * dispatch hidden width; plus E experts, F expert SwiGLU width, the b_x dtype
+ * and H, the model width of a LatentMoE layer (0 = no latent projection). */
+typedef struct {
+    int64_t S;
+    int64_t GBS;
+    int32_t K;
+    int32_t D;
+    int32_t E;
+    int32_t F;
+    int32_t x_dtype;  /* moe_dtype */
+    int32_t H;
+} moe_shape_t;
+
+/* Bytes of scratch the calls below need for this shape (the maximum over all
+ * calls; one workspace may be reused by every call on one stream).  Returns
+ * MOE_OK and writes *bytes, or a shape error. */
+int moe_workspace_size(const moe_shape_t* shape, size_t* bytes);
+
+/* Router (reading R1, R2, R7): logits[T, E] = x[T, Din] . w_router^T (+ bias),
+ * then moe_topk.  bias [E] fp32 is optional (NULL = none) and is added in fp32
+ * after the product.  Din = H when shape->H > 0, else D. */
+int moe_route(const moe_shape_t* shape, const void* x, const void* w_router, const float* bias,
+              float* logits, int32_t* topk_idx, float* topk_prob, void* ws, size_t ws_bytes, void* stream);
+
+/* Top-K of given fp32 logits [T, E], one warp per token: the K largest
+ * logits (ties to the lower expert index), ordered by descending logit, and
+ * renormalised probabilities p_k = exp(z_k - z_max) / sum over the K chosen
+ * (equal to softmax over all E restricted to the chosen set). */
+int moe_topk(const moe_shape_t* shape, const float* logits, int32_t* topk_idx, float* topk_prob, void* stream);
+
+/* Dispatch (forward hidden and probability transfers, Sec. 4.1 footnote):
+ * builds expert_offsets [E+1], row_of_slot [TK] and token_of_row [TK] by a
+ * deterministic counting sort of topk_idx [T, K] (histogram + prefix sum),
+ * then x_perm[row] = x[token_of_row[row]] ([TK, D]) and
+ * prob_perm[row] = topk_prob[slot].  x is the dispatch input [T, D] (for
+ * LatentMoE the down-projected x_lat).  x_perm may be NULL to build only the
+ * permutation and prob_perm.  Expert indices outside [0, E) set the device
+ * status word and are skipped. */
+int moe_dispatch(const moe_shape_t* shape, const void* x, const int32_t* topk_idx, const float* topk_prob,
+                 int32_t* expert_offsets, int32_t* row_of_slot, int32_t* token_of_row,
+                 void* x_perm, float* prob_perm, void* ws, size_t ws_bytes, void* stream);
+
+/* Grouped SwiGLU expert FFN (Sec. 5.2 grouped GEMM; reading R6): for every
+ * expert e and its rows, h = x_perm . w1_e^T ([rows, 2F], packed order),
+ * a = silu(g) * u ([rows, F]), y_perm = a . w2_e^T ([rows, D]).  h_save and
+ * act_save are written for the backward pass.  Reads expert_offsets on the
+ * device (no host synchronisation). */
+int moe_expert_ffn(const moe_shape_t* shape, const void* x_perm, const int32_t* expert_offsets,
+                   const void* w1, const void* w2, void* h_save, void* act_save, void* y_perm,
+                   void* ws, size_t ws_bytes, void* stream);
+
+/* Combine (forward hidden combine, Sec. 4.1 footnote; reading R5):
+ * y[t] = sum_k prob_perm[r] * y_perm[r], r = row_of_slot[t K + k], fp32
+ * accumulation, one rounding to the storage dtype.  y is [T, D]. */
+int moe_combine(const moe_shape_t* shape, const void* y_perm, const float* prob_perm, const int32_t* row_of_slot,
+                void* y, void* stream);
+
+/* Combine backward (inverse of the combine): dy_perm[r] = prob_perm[r] * dy[t]
+ * and dprob_perm[r] = <dy[t], y_perm[r]> (fp32) for every slot (t, k). */
+int moe_combine_bwd(const moe_shape_t* shape, const void* dy, const void* y_perm, const float* prob_perm,
+                    const int32_t* row_of_slot, void* dy_perm, float* dprob_perm, void* stream);
+
+/* Expert FFN backward: dA = dy_perm . w2_e, SwiGLU backward from the saved h
+ * (dg = dA u sigmoid(g) (1 + g (1 - sigmoid(g))), du = dA silu(g)),
+ * dx_perm = dH . w1_e, dw2_e = dy_perm_e^T . a_e, dw1_e = dH_e^T . x_perm_e.
+ * dw1 [E, 2F, D] and dw2 [E, D, F] are fp32 and fully written (zero for an
+ * expert with no rows).  dH [TK, 2F] lives in the workspace. */
+int moe_expert_ffn_bwd(const moe_shape_t* shape, const void* dy_perm, const void* x_perm, const void* h_save,
+                       const void* act_save, const int32_t* expert_offsets, const void* w1, const void* w2,
+                       void* dx_perm, float* dw1, float* dw2, void* ws, size_t ws_bytes, void* stream);
+
+/* Dispatch backward (inverse of the hidden and probability dispatches):
+ * dx[t] = sum_k dx_perm[r] (fp32 accumulation; dx [T, D] is overwritten) and
+ * dtopk_prob[t, k] = dprob_perm[r], r = row_of_slot[t K + k]. */
+int moe_dispatch_bwd(const moe_shape_t* shape, const void* dx_perm, const float* dprob_perm,
+                     const int32_t* row_of_slot, void* dx, float* dtopk_prob, void* stream);
+
+/* Router backward: dlogits[t, j] = p_j (dp_j - sum_k p_k dp_k) for the K
+ * chosen experts, 0 elsewhere ([T, E] fp32, fully written);
+ * dx[T, Din] += dlogits . w_router (accumulated into the existing contents,
+ * one rounding); dw_router [E, Din] = dlogits^T . x (fp32, overwritten).
+ * The logit bias gets no gradient. */
+int moe_route_bwd(const moe_shape_t* shape, const void* x, const void* w_router, const int32_t* topk_idx,
+                  const float* topk_prob, const float* dtopk_prob, void* dx, float* dw_router, float* dlogits,
+                  void* ws, size_t ws_bytes, void* stream);
+
+/* LatentMoE projection (dense, T rows): out[T, n_out] = in[T, n_in] . w^T with
+ * w [n_out, n_in].  Down-projection: n_in = H, n_out = D; up-projection:
+ * n_in = D, n_out = H. */
+int moe_latent_proj(const moe_shape_t* shape, int32_t n_in, int32_t n_out, const void* in, const void* w,
+                    void* out, void* ws, size_t ws_bytes, void* stream);
+
+/* LatentMoE projection backward: din = dout . w (overwritten, or added to the
+ * existing contents when accumulate != 0), dw [n_out, n_in] = dout^T . in
+ * (fp32, overwritten).  din may be NULL to skip it. */
+int moe_latent_proj_bwd(const moe_shape_t* shape, int32_t n_in, int32_t n_out, const void* dout, const void* in,
+                        const void* w, void* din, int32_t accumulate, float* dw, void* ws, size_t ws_bytes,
+                        void* stream);
+
+/* Packs w_gate [E, F, D] and w_up [E, F, D] into w1 [E, 2F, D] (layout above). */
+int moe_pack_w1(const moe_shape_t* shape, const void* w_gate, const void* w_up, void* w1, void* stream);
+
+/* Eq. 1 per-layer logical payload with L_E = 1 and constant 1:
+ * S * GBS * K * (4 D b_x + 2 b_p), b_p = 4.  Host only; 0 on a bad shape. */
+uint64_t moe_eq1_bytes(const moe_shape_t* shape);
+
+/* Synchronises `stream`, then returns MOE_OK, MOE_ERR_DEVICE if the device
+ * status word of the current device is set (and clears it), or MOE_ERR_CUDA.
+ * Off the timed path. */
+int moe_check_device_status(void* stream);
+
+/* Raw device status word of the current device (bit flags, 0 = clean):
+ * 1 = expert index out of range, 2 = a bounded pipeline wait expired. */
+int moe_device_status_word(void* stream, uint32_t* word);
+
+/* Last cudaError_t seen by a call that returned MOE_ERR_CUDA (0 if none). */
+int moe_last_cuda_error(void);
+
+/* Human-readable text for a moe_status. */
+const char* moe_strerror(int status);
+
+/* Library version (major * 10000 + minor * 100 + patch). */
+int moe_version(void);
+
+/* Per-kernel timing.  While enabled, every kernel launch is bracketed by
+ * CUDA events on its launch stream; moe_prof_get reads the accumulated
+ * device time per kernel name (synchronising on the recorded events). */
+int moe_prof_enable(int on);
+int moe_prof_reset(void);
+int moe_prof_count(void);
+int moe_prof_get(int i, const char** name, int* launches, double* total_ms);
+
+/* Kernel launches made by this library since load (all streams). */
+uint64_t moe_launch_count(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MOE_GB300_H */

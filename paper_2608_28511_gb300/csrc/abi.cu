@@ -1,0 +1,784 @@
+// The extern "C" entry points declared in include/moe.h: argument
+// validation, workspace carving, per-device state and the call sequence of
+// each layer stage.  No entry point allocates or synchronises (except
+// moe_check_device_status / moe_device_status_word / moe_prof_get).
+#include <atomic>
+#include <cstring>
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include "common.cuh"
+#include "launch.h"
+
+namespace moe {
+
+// Device status word (one per device that loads the library).
+__device__ uint32_t g_status_word;
+
+namespace {
+
+constexpr int kMaxDevices = 64;
+std::mutex g_mu;
+uint32_t* g_status_ptr[kMaxDevices] = {};
+int g_num_sms[kMaxDevices] = {};
+thread_local int g_last_cuda = 0;
+std::atomic<uint64_t> g_launches{0};
+
+// ---- profiling ------------------------------------------------------------
+struct ProfRec {
+  std::string name;
+  int launches = 0;
+  double total_ms = 0.0;
+  std::vector<std::pair<cudaEvent_t, cudaEvent_t>> pending;
+};
+std::atomic<bool> g_prof_on{false};
+std::mutex g_prof_mu;
+std::vector<ProfRec> g_prof;
+std::vector<cudaEvent_t> g_event_pool;
+struct Open {
+  cudaStream_t s;
+  cudaEvent_t ev;
+};
+thread_local std::vector<Open> g_open;
+
+cudaEvent_t pool_get() {
+  if (g_event_pool.empty()) {
+    for (int i = 0; i < 256; ++i) {
+      cudaEvent_t e;
+      if (cudaEventCreate(&e) != cudaSuccess) break;
+      g_event_pool.push_back(e);
+    }
+    if (g_event_pool.empty()) return nullptr;
+  }
+  cudaEvent_t e = g_event_pool.back();
+  g_event_pool.pop_back();
+  return e;
+}
+
+ProfRec& prof_rec(const char* name) {
+  for (auto& r : g_prof)
+    if (r.name == name) return r;
+  g_prof.push_back(ProfRec{});
+  g_prof.back().name = name;
+  return g_prof.back();
+}
+
+void prof_harvest() {
+  for (auto& r : g_prof) {
+    for (auto& pr : r.pending) {
+      float ms = 0.f;
+      cudaEventSynchronize(pr.second);
+      if (cudaEventElapsedTime(&ms, pr.first, pr.second) == cudaSuccess) r.total_ms += ms;
+      g_event_pool.push_back(pr.first);
+      g_event_pool.push_back(pr.second);
+    }
+    r.pending.clear();
+  }
+}
+
+// ---- per-device context ---------------------------------------------------
+int get_ctx(void* stream, Ctx* c) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess || dev < 0 || dev >= kMaxDevices) {
+    g_last_cuda = (int)e;
+    return MOE_ERR_CUDA;
+  }
+  std::lock_guard<std::mutex> lk(g_mu);
+  if (!g_status_ptr[dev]) {
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_status_word);
+    if (e != cudaSuccess) {
+      g_last_cuda = (int)e;
+      return MOE_ERR_CUDA;
+    }
+    int sms = 0;
+    e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) {
+      g_last_cuda = (int)e;
+      return MOE_ERR_CUDA;
+    }
+    g_status_ptr[dev] = (uint32_t*)p;
+    g_num_sms[dev] = sms;
+  }
+  c->stream = (cudaStream_t)stream;
+  c->err = g_status_ptr[dev];
+  c->num_sms = g_num_sms[dev];
+  c->device = dev;
+  return MOE_OK;
+}
+
+int cuda_status(cudaError_t e) {
+  if (e == cudaSuccess) return MOE_OK;
+  g_last_cuda = (int)e;
+  return MOE_ERR_CUDA;
+}
+
+// ---- validation -----------------------------------------------------------
+struct Dims {
+  int64_t T, TK;
+  int K, D, E, F, H, Din;
+  DType dt;
+  size_t bx;
+};
+
+int check_shape(const moe_shape_t* s, Dims* d) {
+  if (!s) return MOE_ERR_NULL;
+  if (s->x_dtype != MOE_BF16 && s->x_dtype != MOE_F32) return MOE_ERR_DTYPE;
+  if (s->S <= 0 || s->GBS <= 0 || s->K <= 0 || s->D <= 0 || s->E <= 0 || s->F <= 0 || s->H < 0)
+    return MOE_ERR_SHAPE;
+  if (s->K > s->E || s->E > kMaxE || s->K > kMaxK) return MOE_ERR_SHAPE;
+  if (s->D % 64 || s->F % 64 || s->H % 64) return MOE_ERR_SHAPE;
+  if (s->S > (int64_t(1) << 31) || s->GBS > (int64_t(1) << 31)) return MOE_ERR_SHAPE;
+  const int64_t T = s->S * s->GBS;
+  const int64_t TK = T * s->K;
+  if (TK >= (int64_t(1) << 31)) return MOE_ERR_SHAPE;
+  d->T = T;
+  d->TK = TK;
+  d->K = s->K;
+  d->D = s->D;
+  d->E = s->E;
+  d->F = s->F;
+  d->H = s->H;
+  d->Din = s->H ? s->H : s->D;
+  d->dt = s->x_dtype == MOE_BF16 ? DType::BF16 : DType::F32;
+  d->bx = dsize(d->dt);
+  return MOE_OK;
+}
+
+bool aligned(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+
+#define REQUIRE_PTR(p)                     \
+  do {                                     \
+    if (!(p)) return MOE_ERR_NULL;         \
+    if (!aligned(p)) return MOE_ERR_ALIGN; \
+  } while (0)
+#define OPTIONAL_PTR(p)                          \
+  do {                                           \
+    if ((p) && !aligned(p)) return MOE_ERR_ALIGN; \
+  } while (0)
+#define TRY(expr)                    \
+  do {                               \
+    int _st = (expr);                \
+    if (_st != MOE_OK) return _st;   \
+  } while (0)
+#define TRY_CUDA(expr) TRY(cuda_status(expr))
+
+size_t align_up(size_t v) { return (v + 255) & ~size_t(255); }
+
+// Workspace carve-up.  Calls are ordered on one stream, so the regions used by
+// different calls may overlap.
+size_t ws_perm(const Dims& d) { return align_up(perm_workspace_bytes(d.TK, d.E)); }
+size_t ws_ffn_bwd(const Dims& d) { return align_up((size_t)d.TK * 2 * d.F * d.bx); }
+size_t ws_route_bwd(const Dims& d) { return align_up((size_t)d.T * d.E * 2); }
+size_t ws_total(const Dims& d) {
+  size_t m = ws_perm(d);
+  m = std::max(m, ws_ffn_bwd(d));
+  m = std::max(m, ws_route_bwd(d));
+  return m + 256;
+}
+
+// Runs one GEMM on the tensor-core engine when it supports the descriptor,
+// else on the CUDA-core engine.
+cudaError_t gemm(const Ctx& c, const GemmDesc& g, const char* tc_name, const char* simt_name) {
+  if (gemm_tc_supports(g)) return launch_gemm_tc(c, g, tc_name);
+  return launch_gemm_simt(c, g, simt_name);
+}
+
+}  // namespace
+
+void prof_begin(const char* name, cudaStream_t s) {
+  (void)name;
+  if (!g_prof_on.load(std::memory_order_relaxed)) return;
+  std::lock_guard<std::mutex> lk(g_prof_mu);
+  cudaEvent_t e = pool_get();
+  if (!e) return;
+  cudaEventRecord(e, s);
+  g_open.push_back(Open{s, e});
+}
+
+void prof_end(const char* name, cudaStream_t s) {
+  if (!g_prof_on.load(std::memory_order_relaxed)) return;
+  std::lock_guard<std::mutex> lk(g_prof_mu);
+  if (g_open.empty()) return;
+  Open o = g_open.back();
+  g_open.pop_back();
+  cudaEvent_t e = pool_get();
+  if (!e) {
+    g_event_pool.push_back(o.ev);
+    return;
+  }
+  cudaEventRecord(e, s);
+  ProfRec& r = prof_rec(name);
+  r.launches += 1;
+  r.pending.emplace_back(o.ev, e);
+}
+
+void count_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
+
+}  // namespace moe
+
+using namespace moe;
+
+extern "C" {
+
+int moe_version(void) { return 100; }
+
+const char* moe_strerror(int status) {
+  switch (status) {
+    case MOE_OK: return "ok";
+    case MOE_ERR_SHAPE: return "invalid shape (non-positive size, K > E, E > 256, K > 16, D/F/H not a multiple of 64, or T*K >= 2^31)";
+    case MOE_ERR_DTYPE: return "unknown dtype";
+    case MOE_ERR_ALIGN: return "pointer not 16-byte aligned";
+    case MOE_ERR_NULL: return "required pointer is NULL";
+    case MOE_ERR_WORKSPACE: return "workspace smaller than moe_workspace_size()";
+    case MOE_ERR_CUDA: return "CUDA runtime error (see moe_last_cuda_error)";
+    case MOE_ERR_DEVICE: return "device status word set (out-of-range expert index or expired bounded wait)";
+    case MOE_ERR_UNSUPPORTED: return "unsupported request";
+    default: return "unknown status";
+  }
+}
+
+int moe_last_cuda_error(void) { return g_last_cuda; }
+
+uint64_t moe_launch_count(void) { return g_launches.load(); }
+
+int moe_workspace_size(const moe_shape_t* shape, size_t* bytes) {
+  Dims d;
+  TRY(check_shape(shape, &d));
+  if (!bytes) return MOE_ERR_NULL;
+  *bytes = ws_total(d);
+  return MOE_OK;
+}
+
+uint64_t moe_eq1_bytes(const moe_shape_t* shape) {
+  Dims d;
+  if (check_shape(shape, &d) != MOE_OK) return 0;
+  return (uint64_t)shape->S * (uint64_t)shape->GBS * (uint64_t)shape->K *
+         (4ull * (uint64_t)shape->D * (uint64_t)d.bx + 2ull * 4ull);
+}
+
+int moe_topk(const moe_shape_t* shape, const float* logits, int32_t* topk_idx, float* topk_prob, void* stream) {
+  Dims d;
+  TRY(check_shape(shape, &d));
+  REQUIRE_PTR(logits);
+  REQUIRE_PTR(topk_idx);
+  REQUIRE_PTR(topk_prob);
+  Ctx c;
+  TRY(get_ctx(stream, &c));
+  TRY_CUDA(launch_topk(c, logits, d.T, d.E, d.K, topk_idx, topk_prob));
+  return MOE_OK;
+}
+
+int moe_route(const moe_shape_t* shape, const void* x, const void* w_router, const float* bias, float* logits,
+              int32_t* topk_idx, float* topk_prob, void* ws, size_t ws_bytes, void* stream) {
+  Dims d;
+  TRY(check_shape(shape, &d));
+  REQUIRE_PTR(x);
+  REQUIRE_PTR(w_router);
+  OPTIONAL_PTR(bias);
+  REQUIRE_PTR(logits);
+  REQUIRE_PTR(topk_idx);
+  REQUIRE_PTR(topk_prob);
+  (void)ws;
+  (void)ws_bytes;
+  Ctx c;
+  TRY(get_ctx(stream, &c));
+  GemmDesc g;
+  g.group = Group::Dense;
+  g.epi = Epi::StoreBias;
+  g.M = d.T;
+  g.N = d.E;
+  g.K = d.Din;
+  g.A = x;
+  g.a_type = d.dt;
+  g.sa_m = d.Din;
+  g.sa_k = 1;
+  g.B = w_router;
+  g.b_type = d.dt;
+  g.sb_n = d.Din;
+  g.sb_k = 1;
+  g.C = logits;
+  g.c_type = DType::F32;
+  g.ldc = d.E;
+  g.bias = bias;
+  if (d.T > 0) TRY_CUDA(gemm(c, g, "router_gemm_tc", "router_gemm_simt"));
+  TRY_CUDA(launch_topk(c, logits, d.T, d.E, d.K, topk_idx, topk_prob));
+  return MOE_OK;
+}
+
+int moe_dispatch(const moe_shape_t* shape, const void* x, const int32_t* topk_idx, const float* topk_prob,
+                 int32_t* expert_offsets, int32_t* row_of_slot, int32_t* token_of_row, void* x_perm,
+                 float* prob_perm, void* ws, size_t ws_bytes, void* stream) {
+  Dims d;
+  TRY(check_shape(shape, &d));
+  REQUIRE_PTR(topk_idx);
+  REQUIRE_PTR(topk_prob);
+  REQUIRE_PTR(expert_offsets);
+  REQUIRE_PTR(row_of_slot);
+  REQUIRE_PTR(token_of_row);
+  REQUIRE_PTR(prob_perm);
+  REQUIRE_PTR(ws);
+  OPTIONAL_PTR(x_perm);
+  if (x_perm) REQUIRE_PTR(x);
+  if (ws_bytes < ws_perm(d)) return MOE_ERR_WORKSPACE;
+  Ctx c;
+  TRY(get_ctx(stream, &c));
+  TRY_CUDA(launch_permutation(c, topk_idx, topk_prob, d.T, d.K, d.E, expert_offsets, row_of_slot, token_of_row,
+                              prob_perm, ws));
+  if (x_perm) TRY_CUDA(launch_dispatch_rows(c, x, row_of_slot, d.T, d.K, (int64_t)d.D * d.bx, x_perm));
+  return MOE_OK;
+}
+
+int moe_expert_ffn(const moe_shape_t* shape, const void* x_perm, const int32_t* expert_offsets, const void* w1,
+                   const void* w2, void* h_save, void* act_save, void* y_perm, void* ws, size_t ws_bytes,
+                   void* stream) {
+  Dims d;
+  TRY(check_shape(shape, &d));
+  REQUIRE_PTR(x_perm);
+  REQUIRE_PTR(expert_offsets);
+  REQUIRE_PTR(w1);
+  REQUIRE_PTR(w2);
+  REQUIRE_PTR(h_save);
+  REQUIRE_PTR(act_save);
+  REQUIRE_PTR(y_perm);
+  (void)ws;
+  (void)ws_bytes;
+  Ctx c;
+  TRY(get_ctx(stream, &c));
+  if (d.TK == 0) return MOE_OK;
+  // GEMM-1 + fused SwiGLU: h = x_perm . w1_e^T, a = silu(g) * u
+  GemmDesc g1;
+  g1.group = Group::M;
+  g1.epi = Epi::SwigluFwd;
+  g1.N = 2 * d.F;
+  g1.K = d.D;
+  g1.num_groups = d.E;
+  g1.offsets = expert_offsets;
+  g1.max_rows = d.TK;
+  g1.A = x_perm;
+  g1.a_type = d.dt;
+  g1.sa_m = d.D;
+  g1.sa_k = 1;
+  g1.B = w1;
+  g1.b_type = d.dt;
+  g1.sb_n = d.D;
+  g1.sb_k = 1;
+  g1.sb_g = (int64_t)2 * d.F * d.D;
+  g1.C = h_save;
+  g1.c_type = d.dt;
+  g1.ldc = 2 * d.F;
+  g1.aux = act_save;
+  TRY_CUDA(gemm(c, g1, "ffn1_swiglu_tc", "ffn1_swiglu_simt"));
+  // GEMM-2: y_perm = a . w2_e^T
+  GemmDesc g2;
+  g2.group = Group::M;
+  g2.epi = Epi::Store;
+  g2.N = d.D;
+  g2.K = d.F;
+  g2.num_groups = d.E;
+  g2.offsets = expert_offsets;
+  g2.max_rows = d.TK;
+  g2.A = act_save;
+  g2.a_type = d.dt;
+  g2.sa_m = d.F;
+  g2.sa_k = 1;
+  g2.B = w2;
+  g2.b_type = d.dt;
+  g2.sb_n = d.F;
+  g2.sb_k = 1;
+  g2.sb_g = (int64_t)d.D * d.F;
+  g2.C = y_perm;
+  g2.c_type = d.dt;
+  g2.ldc = d.D;
+  TRY_CUDA(gemm(c, g2, "ffn2_tc", "ffn2_simt"));
+  return MOE_OK;
+}
+
+int moe_combine(const moe_shape_t* shape, const void* y_perm, const float* prob_perm, const int32_t* row_of_slot,
+                void* y, void* stream) {
+  Dims d;
+  TRY(check_shape(shape, &d));
+  REQUIRE_PTR(y_perm);
+  REQUIRE_PTR(prob_perm);
+  REQUIRE_PTR(row_of_slot);
+  REQUIRE_PTR(y);
+  Ctx c;
+  TRY(get_ctx(stream, &c));
+  TRY_CUDA(launch_combine(c, d.dt, y_perm, prob_perm, row_of_slot, d.T, d.K, d.D, y));
+  return MOE_OK;
+}
+
+int moe_combine_bwd(const moe_shape_t* shape, const void* dy, const void* y_perm, const float* prob_perm,
+                    const int32_t* row_of_slot, void* dy_perm, float* dprob_perm, void* stream) {
+  Dims d;
+  TRY(check_shape(shape, &d));
+  REQUIRE_PTR(dy);
+  REQUIRE_PTR(y_perm);
+  REQUIRE_PTR(prob_perm);
+  REQUIRE_PTR(row_of_slot);
+  REQUIRE_PTR(dy_perm);
+  REQUIRE_PTR(dprob_perm);
+  Ctx c;
+  TRY(get_ctx(stream, &c));
+  TRY_CUDA(launch_combine_bwd(c, d.dt, dy, y_perm, prob_perm, row_of_slot, d.T, d.K, d.D, dy_perm, dprob_perm));
+  return MOE_OK;
+}
+
+int moe_expert_ffn_bwd(const moe_shape_t* shape, const void* dy_perm, const void* x_perm, const void* h_save,
+                       const void* act_save, const int32_t* expert_offsets, const void* w1, const void* w2,
+                       void* dx_perm, float* dw1, float* dw2, void* ws, size_t ws_bytes, void* stream) {
+  Dims d;
+  TRY(check_shape(shape, &d));
+  REQUIRE_PTR(dy_perm);
+  REQUIRE_PTR(x_perm);
+  REQUIRE_PTR(h_save);
+  REQUIRE_PTR(act_save);
+  REQUIRE_PTR(expert_offsets);
+  REQUIRE_PTR(w1);
+  REQUIRE_PTR(w2);
+  REQUIRE_PTR(dx_perm);
+  REQUIRE_PTR(dw1);
+  REQUIRE_PTR(dw2);
+  REQUIRE_PTR(ws);
+  if (ws_bytes < ws_ffn_bwd(d)) return MOE_ERR_WORKSPACE;
+  Ctx c;
+  TRY(get_ctx(stream, &c));
+  void* dH = ws;
+  // dgrad-2 with the SwiGLU backward epilogue: dA = dy_perm . w2_e -> dH
+  GemmDesc a;
+  a.group = Group::M;
+  a.epi = Epi::SwigluBwd;
+  a.N = d.F;
+  a.K = d.D;
+  a.num_groups = d.E;
+  a.offsets = expert_offsets;
+  a.max_rows = d.TK;
+  a.A = dy_perm;
+  a.a_type = d.dt;
+  a.sa_m = d.D;
+  a.sa_k = 1;
+  a.B = w2;
+  a.b_type = d.dt;
+  a.sb_n = 1;
+  a.sb_k = d.F;
+  a.sb_g = (int64_t)d.D * d.F;
+  a.C = dH;
+  a.c_type = d.dt;
+  a.ldc = 2 * d.F;
+  a.h_in = h_save;
+  // wgrad-2: dw2_e[d, f] = sum_rows dy_perm[r, d] a[r, f]
+  GemmDesc b;
+  b.group = Group::K;
+  b.epi = Epi::Store;
+  b.M = d.D;
+  b.N = d.F;
+  b.num_groups = d.E;
+  b.offsets = expert_offsets;
+  b.A = dy_perm;
+  b.a_type = d.dt;
+  b.sa_m = 1;
+  b.sa_k = d.D;
+  b.B = act_save;
+  b.b_type = d.dt;
+  b.sb_n = 1;
+  b.sb_k = d.F;
+  b.C = dw2;
+  b.c_type = DType::F32;
+  b.ldc = d.F;
+  b.sc_g = (int64_t)d.D * d.F;
+  // dgrad-1: dx_perm = dH . w1_e
+  GemmDesc cg;
+  cg.group = Group::M;
+  cg.epi = Epi::Store;
+  cg.N = d.D;
+  cg.K = 2 * d.F;
+  cg.num_groups = d.E;
+  cg.offsets = expert_offsets;
+  cg.max_rows = d.TK;
+  cg.A = dH;
+  cg.a_type = d.dt;
+  cg.sa_m = 2 * d.F;
+  cg.sa_k = 1;
+  cg.B = w1;
+  cg.b_type = d.dt;
+  cg.sb_n = 1;
+  cg.sb_k = d.D;
+  cg.sb_g = (int64_t)2 * d.F * d.D;
+  cg.C = dx_perm;
+  cg.c_type = d.dt;
+  cg.ldc = d.D;
+  // wgrad-1: dw1_e[j, d] = sum_rows dH[r, j] x_perm[r, d]
+  GemmDesc w;
+  w.group = Group::K;
+  w.epi = Epi::Store;
+  w.M = 2 * d.F;
+  w.N = d.D;
+  w.num_groups = d.E;
+  w.offsets = expert_offsets;
+  w.A = dH;
+  w.a_type = d.dt;
+  w.sa_m = 1;
+  w.sa_k = 2 * d.F;
+  w.B = x_perm;
+  w.b_type = d.dt;
+  w.sb_n = 1;
+  w.sb_k = d.D;
+  w.C = dw1;
+  w.c_type = DType::F32;
+  w.ldc = d.D;
+  w.sc_g = (int64_t)2 * d.F * d.D;
+  if (d.TK > 0) TRY_CUDA(gemm(c, a, "ffn2_dgrad_swiglu_tc", "ffn2_dgrad_swiglu_simt"));
+  TRY_CUDA(gemm(c, b, "ffn2_wgrad_tc", "ffn2_wgrad_simt"));
+  if (d.TK > 0) TRY_CUDA(gemm(c, cg, "ffn1_dgrad_tc", "ffn1_dgrad_simt"));
+  TRY_CUDA(gemm(c, w, "ffn1_wgrad_tc", "ffn1_wgrad_simt"));
+  return MOE_OK;
+}
+
+int moe_dispatch_bwd(const moe_shape_t* shape, const void* dx_perm, const float* dprob_perm,
+                     const int32_t* row_of_slot, void* dx, float* dtopk_prob, void* stream) {
+  Dims d;
+  TRY(check_shape(shape, &d));
+  REQUIRE_PTR(dx_perm);
+  REQUIRE_PTR(dprob_perm);
+  REQUIRE_PTR(row_of_slot);
+  REQUIRE_PTR(dx);
+  REQUIRE_PTR(dtopk_prob);
+  Ctx c;
+  TRY(get_ctx(stream, &c));
+  TRY_CUDA(launch_dispatch_bwd(c, d.dt, dx_perm, dprob_perm, row_of_slot, d.T, d.K, d.D, dx, dtopk_prob));
+  return MOE_OK;
+}
+
+int moe_route_bwd(const moe_shape_t* shape, const void* x, const void* w_router, const int32_t* topk_idx,
+                  const float* topk_prob, const float* dtopk_prob, void* dx, float* dw_router, float* dlogits,
+                  void* ws, size_t ws_bytes, void* stream) {
+  Dims d;
+  TRY(check_shape(shape, &d));
+  REQUIRE_PTR(x);
+  REQUIRE_PTR(w_router);
+  REQUIRE_PTR(topk_idx);
+  REQUIRE_PTR(topk_prob);
+  REQUIRE_PTR(dtopk_prob);
+  REQUIRE_PTR(dx);
+  REQUIRE_PTR(dw_router);
+  REQUIRE_PTR(dlogits);
+  REQUIRE_PTR(ws);
+  if (ws_bytes < ws_route_bwd(d)) return MOE_ERR_WORKSPACE;
+  Ctx c;
+  TRY(get_ctx(stream, &c));
+  void* dz16 = d.dt == DType::BF16 ? ws : nullptr;
+  TRY_CUDA(launch_route_dz(c, topk_idx, topk_prob, dtopk_prob, d.T, d.E, d.K, dlogits, dz16));
+  // dx += dz . w_router   (M = T, N = Din, K = E)
+  GemmDesc a;
+  a.group = Group::Dense;
+  a.epi = Epi::Accum;
+  a.M = d.T;
+  a.N = d.Din;
+  a.K = d.E;
+  a.A = dlogits;
+  a.a_type = DType::F32;
+  a.sa_m = d.E;
+  a.sa_k = 1;
+  a.B = w_router;
+  a.b_type = d.dt;
+  a.sb_n = 1;
+  a.sb_k = d.Din;
+  a.C = dx;
+  a.c_type = d.dt;
+  a.ldc = d.Din;
+  // dw_router = dz^T . x   (M = E, N = Din, K = T)
+  GemmDesc b;
+  b.group = Group::Dense;
+  b.epi = Epi::Store;
+  b.M = d.E;
+  b.N = d.Din;
+  b.K = d.T;
+  b.A = dlogits;
+  b.a_type = DType::F32;
+  b.sa_m = 1;
+  b.sa_k = d.E;
+  b.B = x;
+  b.b_type = d.dt;
+  b.sb_n = 1;
+  b.sb_k = d.Din;
+  b.C = dw_router;
+  b.c_type = DType::F32;
+  b.ldc = d.Din;
+  if (d.dt == DType::BF16) {
+    // tensor-core path reads the bf16 copy of dz
+    GemmDesc a16 = a, b16 = b;
+    a16.A = dz16;
+    a16.a_type = DType::BF16;
+    b16.A = dz16;
+    b16.a_type = DType::BF16;
+    if (gemm_tc_supports(a16)) a = a16;
+    if (gemm_tc_supports(b16)) b = b16;
+  }
+  if (d.T > 0) TRY_CUDA(gemm(c, a, "router_dgrad_tc", "router_dgrad_simt"));
+  TRY_CUDA(gemm(c, b, "router_wgrad_tc", "router_wgrad_simt"));
+  return MOE_OK;
+}
+
+int moe_latent_proj(const moe_shape_t* shape, int32_t n_in, int32_t n_out, const void* in, const void* w,
+                    void* out, void* ws, size_t ws_bytes, void* stream) {
+  Dims d;
+  TRY(check_shape(shape, &d));
+  if (n_in <= 0 || n_out <= 0 || n_in % 64 || n_out % 64) return MOE_ERR_SHAPE;
+  REQUIRE_PTR(in);
+  REQUIRE_PTR(w);
+  REQUIRE_PTR(out);
+  (void)ws;
+  (void)ws_bytes;
+  Ctx c;
+  TRY(get_ctx(stream, &c));
+  GemmDesc g;
+  g.group = Group::Dense;
+  g.epi = Epi::Store;
+  g.M = d.T;
+  g.N = n_out;
+  g.K = n_in;
+  g.A = in;
+  g.a_type = d.dt;
+  g.sa_m = n_in;
+  g.sa_k = 1;
+  g.B = w;
+  g.b_type = d.dt;
+  g.sb_n = n_in;
+  g.sb_k = 1;
+  g.C = out;
+  g.c_type = d.dt;
+  g.ldc = n_out;
+  if (d.T > 0) TRY_CUDA(gemm(c, g, "latent_fwd_tc", "latent_fwd_simt"));
+  return MOE_OK;
+}
+
+int moe_latent_proj_bwd(const moe_shape_t* shape, int32_t n_in, int32_t n_out, const void* dout, const void* in,
+                        const void* w, void* din, int32_t accumulate, float* dw, void* ws, size_t ws_bytes,
+                        void* stream) {
+  Dims d;
+  TRY(check_shape(shape, &d));
+  if (n_in <= 0 || n_out <= 0 || n_in % 64 || n_out % 64) return MOE_ERR_SHAPE;
+  REQUIRE_PTR(dout);
+  REQUIRE_PTR(in);
+  REQUIRE_PTR(w);
+  REQUIRE_PTR(dw);
+  OPTIONAL_PTR(din);
+  (void)ws;
+  (void)ws_bytes;
+  Ctx c;
+  TRY(get_ctx(stream, &c));
+  if (din && d.T > 0) {
+    // din = dout . w   (M = T, N = n_in, K = n_out)
+    GemmDesc a;
+    a.group = Group::Dense;
+    a.epi = accumulate ? Epi::Accum : Epi::Store;
+    a.M = d.T;
+    a.N = n_in;
+    a.K = n_out;
+    a.A = dout;
+    a.a_type = d.dt;
+    a.sa_m = n_out;
+    a.sa_k = 1;
+    a.B = w;
+    a.b_type = d.dt;
+    a.sb_n = 1;
+    a.sb_k = n_in;
+    a.C = din;
+    a.c_type = d.dt;
+    a.ldc = n_in;
+    TRY_CUDA(gemm(c, a, "latent_dgrad_tc", "latent_dgrad_simt"));
+  }
+  // dw = dout^T . in   (M = n_out, N = n_in, K = T)
+  GemmDesc b;
+  b.group = Group::Dense;
+  b.epi = Epi::Store;
+  b.M = n_out;
+  b.N = n_in;
+  b.K = d.T;
+  b.A = dout;
+  b.a_type = d.dt;
+  b.sa_m = 1;
+  b.sa_k = n_out;
+  b.B = in;
+  b.b_type = d.dt;
+  b.sb_n = 1;
+  b.sb_k = n_in;
+  b.C = dw;
+  b.c_type = DType::F32;
+  b.ldc = n_in;
+  TRY_CUDA(gemm(c, b, "latent_wgrad_tc", "latent_wgrad_simt"));
+  return MOE_OK;
+}
+
+int moe_pack_w1(const moe_shape_t* shape, const void* w_gate, const void* w_up, void* w1, void* stream) {
+  Dims d;
+  TRY(check_shape(shape, &d));
+  REQUIRE_PTR(w_gate);
+  REQUIRE_PTR(w_up);
+  REQUIRE_PTR(w1);
+  Ctx c;
+  TRY(get_ctx(stream, &c));
+  TRY_CUDA(launch_pack_w1(c, d.dt, w_gate, w_up, d.E, d.F, d.D, w1));
+  return MOE_OK;
+}
+
+int moe_device_status_word(void* stream, uint32_t* word) {
+  if (!word) return MOE_ERR_NULL;
+  Ctx c;
+  TRY(get_ctx(stream, &c));
+  TRY_CUDA(cudaStreamSynchronize(c.stream));
+  TRY_CUDA(cudaMemcpy(word, c.err, sizeof(uint32_t), cudaMemcpyDeviceToHost));
+  return MOE_OK;
+}
+
+int moe_check_device_status(void* stream) {
+  uint32_t w = 0;
+  TRY(moe_device_status_word(stream, &w));
+  if (w) {
+    Ctx c;
+    TRY(get_ctx(stream, &c));
+    TRY_CUDA(cudaMemsetAsync(c.err, 0, sizeof(uint32_t), c.stream));
+    TRY_CUDA(cudaStreamSynchronize(c.stream));
+    return MOE_ERR_DEVICE;
+  }
+  return MOE_OK;
+}
+
+int moe_prof_enable(int on) {
+  std::lock_guard<std::mutex> lk(g_prof_mu);
+  if (on && g_event_pool.empty()) {
+    for (int i = 0; i < 1024; ++i) {
+      cudaEvent_t e;
+      if (cudaEventCreate(&e) != cudaSuccess) break;
+      g_event_pool.push_back(e);
+    }
+  }
+  g_prof_on.store(on != 0);
+  return MOE_OK;
+}
+
+int moe_prof_reset(void) {
+  std::lock_guard<std::mutex> lk(g_prof_mu);
+  prof_harvest();
+  g_prof.clear();
+  return MOE_OK;
+}
+
+int moe_prof_count(void) {
+  std::lock_guard<std::mutex> lk(g_prof_mu);
+  return (int)g_prof.size();
+}
+
+int moe_prof_get(int i, const char** name, int* launches, double* total_ms) {
+  std::lock_guard<std::mutex> lk(g_prof_mu);
+  prof_harvest();
+  if (i < 0 || i >= (int)g_prof.size()) return MOE_ERR_SHAPE;
+  if (name) *name = g_prof[i].name.c_str();
+  if (launches) *launches = g_prof[i].launches;
+  if (total_ms) *total_ms = g_prof[i].total_ms;
+  return MOE_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,108 @@
+// Internal launcher interface between the C ABI (abi.cu) and the kernels.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+#include <stddef.h>
+
+namespace moe {
+
+struct Ctx {
+  cudaStream_t stream;
+  uint32_t* err;   // device status word of the current device
+  int num_sms;
+  int device;
+};
+
+// Per-kernel CUDA-event timing and launch counting (implemented in abi.cu).
+void prof_begin(const char* name, cudaStream_t s);
+void prof_end(const char* name, cudaStream_t s);
+void count_launch();
+
+struct KernelScope {
+  const char* name;
+  cudaStream_t s;
+  KernelScope(const char* n, cudaStream_t st) : name(n), s(st) { prof_begin(name, s); }
+  ~KernelScope() { prof_end(name, s); count_launch(); }
+};
+
+enum class DType : int { BF16 = 0, F32 = 1 };
+
+inline size_t dsize(DType t) { return t == DType::BF16 ? 2 : 4; }
+
+// ---------------------------------------------------------------------------
+// router.cu
+// ---------------------------------------------------------------------------
+constexpr int kMaxK = 16;
+constexpr int kMaxE = 256;
+
+cudaError_t launch_topk(const Ctx& c, const float* logits, int64_t T, int E, int K, int32_t* idx, float* prob);
+// dz[T, E] fp32 (fully written) and optionally a bf16 copy.
+cudaError_t launch_route_dz(const Ctx& c, const int32_t* idx, const float* prob, const float* dprob, int64_t T,
+                            int E, int K, float* dz, void* dz_bf16);
+
+// ---------------------------------------------------------------------------
+// permute.cu
+// ---------------------------------------------------------------------------
+size_t perm_workspace_bytes(int64_t TK, int E);
+cudaError_t launch_permutation(const Ctx& c, const int32_t* idx, const float* prob, int64_t T, int K, int E,
+                               int32_t* offsets, int32_t* row_of_slot, int32_t* token_of_row, float* prob_perm,
+                               void* ws);
+cudaError_t launch_dispatch_rows(const Ctx& c, const void* x, const int32_t* row_of_slot, int64_t T, int K,
+                                 int64_t row_bytes, void* x_perm);
+cudaError_t launch_combine(const Ctx& c, DType dt, const void* y_perm, const float* prob_perm,
+                           const int32_t* row_of_slot, int64_t T, int K, int D, void* y);
+cudaError_t launch_combine_bwd(const Ctx& c, DType dt, const void* dy, const void* y_perm, const float* prob_perm,
+                               const int32_t* row_of_slot, int64_t T, int K, int D, void* dy_perm,
+                               float* dprob_perm);
+cudaError_t launch_dispatch_bwd(const Ctx& c, DType dt, const void* dx_perm, const float* dprob_perm,
+                                const int32_t* row_of_slot, int64_t T, int K, int D, void* dx, float* dprob);
+cudaError_t launch_pack_w1(const Ctx& c, DType dt, const void* w_gate, const void* w_up, int E, int F, int D,
+                           void* w1);
+
+// ---------------------------------------------------------------------------
+// Grouped GEMM  C(m, n) = sum_k A(m, k) B(n, k), fp32 accumulation.
+// ---------------------------------------------------------------------------
+enum class Group : int {
+  Dense = 0,  // one problem: M x N x K
+  M = 1,      // group g owns rows [offsets[g], offsets[g+1]) of A and C; B advanced by g * sb_g
+  K = 2,      // group g reduces over k in [offsets[g], offsets[g+1]); C advanced by g * sc_g
+};
+
+enum class Epi : int {
+  Store = 0,      // C = acc
+  StoreBias = 1,  // C = acc + bias[n]
+  Accum = 2,      // C = C + acc
+  SwigluFwd = 3,  // acc is h (packed gate/up, N = 2F): C = h, aux[m, f] = silu(g) u  (aux ld = N/2)
+  SwigluBwd = 4,  // acc is dA (N = F): reads h_in [m, 2F], writes C = dH [m, 2F] (ldc = 2F)
+};
+
+struct GemmDesc {
+  Group group = Group::Dense;
+  Epi epi = Epi::Store;
+  int64_t M = 0, N = 0, K = 0;  // the grouped dimension is taken from offsets
+  int num_groups = 1;
+  const int32_t* offsets = nullptr;  // [num_groups + 1], device
+  int64_t max_rows = 0;              // Group::M: total rows (upper bound for the grid)
+  const void* A = nullptr;
+  DType a_type = DType::BF16;
+  int64_t sa_m = 0, sa_k = 0;        // element strides of A(m, k)
+  const void* B = nullptr;
+  DType b_type = DType::BF16;
+  int64_t sb_n = 0, sb_k = 0, sb_g = 0;
+  void* C = nullptr;
+  DType c_type = DType::BF16;
+  int64_t ldc = 0, sc_g = 0;
+  const float* bias = nullptr;       // StoreBias
+  const void* h_in = nullptr;        // SwigluBwd (c_type)
+  void* aux = nullptr;               // SwigluFwd activation output (c_type)
+};
+
+cudaError_t launch_gemm_simt(const Ctx& c, const GemmDesc& d, const char* name);
+
+// tcgen05 / TMA engine (bf16 operands only).  Returns cudaErrorNotSupported
+// for a descriptor it does not handle.
+bool gemm_tc_supports(const GemmDesc& d);
+cudaError_t launch_gemm_tc(const Ctx& c, const GemmDesc& d, const char* name);
+
+}  // namespace moe

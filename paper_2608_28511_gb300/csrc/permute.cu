@@ -1,0 +1,389 @@
+// Permute family: deterministic counting sort of the routed slots into the
+// expert-grouped order (histogram + prefix sum + in-order ranking), and the
+// in-HBM dispatch / combine and their backward passes.  On one GPU these
+// replace the paper's six expert-parallel transfers per layer (Sec. 4.1
+// footnote).  All row copies use 16-byte vectors, one warp per token.
+#include "common.cuh"
+#include "launch.h"
+
+namespace moe {
+
+constexpr int kChunk = 2048;       // slots per counting-sort chunk
+constexpr int kRankWarps = 8;      // sub-chunks of kChunk / kRankWarps slots
+constexpr int kSub = kChunk / kRankWarps;
+
+static inline int64_t num_chunks(int64_t TK) { return (TK + kChunk - 1) / kChunk; }
+
+size_t perm_workspace_bytes(int64_t TK, int E) {
+  return (size_t)2 * (size_t)E * (size_t)num_chunks(TK) * sizeof(int32_t);
+}
+
+// Per-chunk expert histogram (shared-memory counters; counts are order-free,
+// so the result is deterministic).  Layout: counts[e * nchunks + chunk].
+__global__ void __launch_bounds__(256) perm_hist_kernel(const int32_t* __restrict__ idx, int64_t TK, int E,
+                                                        int nchunks, int32_t* __restrict__ counts, uint32_t* err) {
+  __shared__ int h[kMaxE];
+  for (int i = threadIdx.x; i < E; i += blockDim.x) h[i] = 0;
+  __syncthreads();
+  const int64_t s0 = (int64_t)blockIdx.x * kChunk;
+  const int64_t s1 = min(TK, s0 + kChunk);
+  for (int64_t s = s0 + threadIdx.x; s < s1; s += blockDim.x) {
+    const int e = idx[s];
+    if (e >= 0 && e < E) atomicAdd(&h[e], 1);
+    else set_error(err, kErrIndex);
+  }
+  __syncthreads();
+  for (int i = threadIdx.x; i < E; i += blockDim.x) counts[(int64_t)i * nchunks + blockIdx.x] = h[i];
+}
+
+// Exclusive prefix sum over the expert-major (expert, chunk) table, one block.
+// base[e * nchunks + c] = first row of expert e's slots from chunk c;
+// offsets[e] = base[e * nchunks], offsets[E] = number of valid slots.
+__global__ void __launch_bounds__(1024) perm_scan_kernel(const int32_t* __restrict__ counts, int E, int nchunks,
+                                                         int32_t* __restrict__ base, int32_t* __restrict__ offsets) {
+  __shared__ int part[1024];
+  const int n = E * nchunks;
+  const int per = (n + 1023) / 1024;
+  const int beg = min(n, threadIdx.x * per), end = min(n, beg + per);
+  int sum = 0;
+  for (int i = beg; i < end; ++i) sum += counts[i];
+  part[threadIdx.x] = sum;
+  __syncthreads();
+  for (int off = 1; off < 1024; off <<= 1) {
+    const int v = threadIdx.x >= off ? part[threadIdx.x - off] : 0;
+    __syncthreads();
+    part[threadIdx.x] += v;
+    __syncthreads();
+  }
+  int run = threadIdx.x ? part[threadIdx.x - 1] : 0;
+  for (int i = beg; i < end; ++i) {
+    base[i] = run;
+    run += counts[i];
+  }
+  __syncthreads();
+  for (int e = threadIdx.x; e < E; e += 1024) offsets[e] = base[(int64_t)e * nchunks];
+  if (threadIdx.x == 0) offsets[E] = part[1023];
+}
+
+// Ranks every slot of one chunk in slot order (= token order within an
+// expert, since a token picks an expert at most once), so the permutation is
+// stable in t and bit-reproducible.  Warp w owns slots [w * kSub, (w+1) * kSub)
+// of the chunk and walks them 32 at a time; lanes that share an expert get
+// consecutive rows by __match_any_sync rank.  Also writes prob_perm.
+__global__ void __launch_bounds__(kRankWarps * 32) perm_rank_kernel(
+    const int32_t* __restrict__ idx, const float* __restrict__ prob, int64_t TK, int K, int E, int nchunks,
+    const int32_t* __restrict__ base, int32_t* __restrict__ row_of_slot, int32_t* __restrict__ token_of_row,
+    float* __restrict__ prob_perm) {
+  __shared__ int cnt[kRankWarps * kMaxE];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (int i = threadIdx.x; i < kRankWarps * E; i += blockDim.x) cnt[i] = 0;
+  __syncthreads();
+  const int64_t c0 = (int64_t)blockIdx.x * kChunk;
+  const int64_t w0 = c0 + (int64_t)warp * kSub;
+  const int64_t w1 = min(TK, w0 + kSub);
+  for (int64_t s = w0 + lane; s < w1; s += 32) {
+    const int e = idx[s];
+    if (e >= 0 && e < E) atomicAdd(&cnt[warp * E + e], 1);
+  }
+  __syncthreads();
+  for (int e = threadIdx.x; e < E; e += blockDim.x) {
+    int run = base[(int64_t)e * nchunks + blockIdx.x];
+    for (int w = 0; w < kRankWarps; ++w) {
+      const int c = cnt[w * E + e];
+      cnt[w * E + e] = run;
+      run += c;
+    }
+  }
+  __syncthreads();
+  const unsigned lt = (1u << lane) - 1u;
+  for (int64_t b = w0; b < w0 + kSub; b += 32) {
+    const int64_t s = b + lane;
+    int e = -1;
+    if (s < w1) e = idx[s];
+    const bool valid = (s < w1) && e >= 0 && e < E;
+    const unsigned peers = __match_any_sync(0xffffffffu, valid ? e : -1);
+    const int rank = __popc(peers & lt);
+    const int here = valid ? cnt[warp * E + e] : 0;
+    __syncwarp();
+    if (valid) {
+      const int row = here + rank;
+      row_of_slot[s] = row;
+      token_of_row[row] = (int32_t)(s / K);
+      prob_perm[row] = prob[s];
+      if (rank == __popc(peers) - 1) cnt[warp * E + e] = here + __popc(peers);
+    } else if (s < w1) {
+      row_of_slot[s] = 0;  // keeps downstream gathers in bounds; the status word is set
+    }
+    __syncwarp();
+  }
+}
+
+cudaError_t launch_permutation(const Ctx& c, const int32_t* idx, const float* prob, int64_t T, int K, int E,
+                               int32_t* offsets, int32_t* row_of_slot, int32_t* token_of_row, float* prob_perm,
+                               void* ws) {
+  const int64_t TK = T * K;
+  const int nch = (int)num_chunks(TK);
+  int32_t* counts = (int32_t*)ws;
+  int32_t* base = counts + (int64_t)E * nch;
+  if (TK == 0) {
+    KernelScope ks("perm_zero", c.stream);
+    return cudaMemsetAsync(offsets, 0, sizeof(int32_t) * (E + 1), c.stream);
+  }
+  {
+    KernelScope ks("perm_hist", c.stream);
+    perm_hist_kernel<<<nch, 256, 0, c.stream>>>(idx, TK, E, nch, counts, c.err);
+  }
+  cudaError_t st = cudaGetLastError();
+  if (st != cudaSuccess) return st;
+  {
+    KernelScope ks("perm_scan", c.stream);
+    perm_scan_kernel<<<1, 1024, 0, c.stream>>>(counts, E, nch, base, offsets);
+  }
+  st = cudaGetLastError();
+  if (st != cudaSuccess) return st;
+  {
+    KernelScope ks("perm_rank", c.stream);
+    perm_rank_kernel<<<nch, kRankWarps * 32, 0, c.stream>>>(idx, prob, TK, K, E, nch, base, row_of_slot,
+                                                            token_of_row, prob_perm);
+  }
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// Row movers: one warp per token, lanes stride over the row's 16-byte vectors.
+// ---------------------------------------------------------------------------
+
+__device__ __forceinline__ void load_rows(const int32_t* __restrict__ row_of_slot, int64_t t, int K,
+                                          int32_t (&rows)[kMaxK]) {
+#pragma unroll
+  for (int k = 0; k < kMaxK; ++k) rows[k] = (k < K) ? __ldg(row_of_slot + t * K + k) : 0;
+}
+
+// Dispatch: each token's row is read once and written to its K rows.
+__global__ void __launch_bounds__(256) dispatch_rows_kernel(const uint4* __restrict__ x,
+                                                            const int32_t* __restrict__ row_of_slot, int64_t T,
+                                                            int K, int vpr, uint4* __restrict__ x_perm) {
+  const int lane = threadIdx.x & 31;
+  const int64_t t = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  if (t >= T) return;
+  int32_t rows[kMaxK];
+  load_rows(row_of_slot, t, K, rows);
+  const uint4* src = x + t * vpr;
+  for (int v = lane; v < vpr; v += 32) {
+    const uint4 val = ld_stream(src + v);
+#pragma unroll
+    for (int k = 0; k < kMaxK; ++k)
+      if (k < K) st_stream(x_perm + (int64_t)rows[k] * vpr + v, val);
+  }
+}
+
+cudaError_t launch_dispatch_rows(const Ctx& c, const void* x, const int32_t* row_of_slot, int64_t T, int K,
+                                 int64_t row_bytes, void* x_perm) {
+  if (T == 0) return cudaSuccess;
+  const int warps = 8;
+  KernelScope ks("dispatch_rows", c.stream);
+  dispatch_rows_kernel<<<(unsigned)((T + warps - 1) / warps), 32 * warps, 0, c.stream>>>(
+      (const uint4*)x, row_of_slot, T, K, (int)(row_bytes / 16), (uint4*)x_perm);
+  return cudaGetLastError();
+}
+
+// Combine: y[t] = sum_k p_k Y_perm[row_k], fp32 accumulation, one rounding.
+template <typename T>
+__global__ void __launch_bounds__(256) combine_kernel(const uint4* __restrict__ y_perm,
+                                                      const float* __restrict__ prob_perm,
+                                                      const int32_t* __restrict__ row_of_slot, int64_t Tn, int K,
+                                                      int vpr, uint4* __restrict__ y) {
+  constexpr int NV = Vec<T>::N;
+  const int lane = threadIdx.x & 31;
+  const int64_t t = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  if (t >= Tn) return;
+  int32_t rows[kMaxK];
+  load_rows(row_of_slot, t, K, rows);
+  float p[kMaxK];
+#pragma unroll
+  for (int k = 0; k < kMaxK; ++k) p[k] = (k < K) ? __ldg(prob_perm + rows[k]) : 0.f;
+  for (int v = lane; v < vpr; v += 32) {
+    float acc[NV];
+#pragma unroll
+    for (int i = 0; i < NV; ++i) acc[i] = 0.f;
+    uint4 raw[kMaxK];
+#pragma unroll
+    for (int k = 0; k < kMaxK; ++k)
+      if (k < K) raw[k] = ld_stream(y_perm + (int64_t)rows[k] * vpr + v);
+#pragma unroll
+    for (int k = 0; k < kMaxK; ++k) {
+      if (k < K) {
+        float f[NV];
+        unpack16<T>(raw[k], f);
+#pragma unroll
+        for (int i = 0; i < NV; ++i) acc[i] = fmaf(p[k], f[i], acc[i]);
+      }
+    }
+    st_stream(y + t * vpr + v, pack16<T>(acc));
+  }
+}
+
+cudaError_t launch_combine(const Ctx& c, DType dt, const void* y_perm, const float* prob_perm,
+                           const int32_t* row_of_slot, int64_t T, int K, int D, void* y) {
+  if (T == 0) return cudaSuccess;
+  const int warps = 8;
+  const int vpr = (int)((int64_t)D * dsize(dt) / 16);
+  const unsigned grid = (unsigned)((T + warps - 1) / warps);
+  KernelScope ks("combine", c.stream);
+  if (dt == DType::BF16)
+    combine_kernel<bf16><<<grid, 32 * warps, 0, c.stream>>>((const uint4*)y_perm, prob_perm, row_of_slot, T, K,
+                                                            vpr, (uint4*)y);
+  else
+    combine_kernel<float><<<grid, 32 * warps, 0, c.stream>>>((const uint4*)y_perm, prob_perm, row_of_slot, T, K,
+                                                             vpr, (uint4*)y);
+  return cudaGetLastError();
+}
+
+// Combine backward: dY_perm[row_k] = p_k dy[t]; dprob_perm[row_k] = <dy[t], Y_perm[row_k]>.
+template <typename T>
+__global__ void __launch_bounds__(256) combine_bwd_kernel(const uint4* __restrict__ dy,
+                                                          const uint4* __restrict__ y_perm,
+                                                          const float* __restrict__ prob_perm,
+                                                          const int32_t* __restrict__ row_of_slot, int64_t Tn,
+                                                          int K, int vpr, uint4* __restrict__ dy_perm,
+                                                          float* __restrict__ dprob_perm) {
+  constexpr int NV = Vec<T>::N;
+  const int lane = threadIdx.x & 31;
+  const int64_t t = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  if (t >= Tn) return;
+  int32_t rows[kMaxK];
+  load_rows(row_of_slot, t, K, rows);
+  float p[kMaxK], dot[kMaxK];
+#pragma unroll
+  for (int k = 0; k < kMaxK; ++k) {
+    p[k] = (k < K) ? __ldg(prob_perm + rows[k]) : 0.f;
+    dot[k] = 0.f;
+  }
+  for (int v = lane; v < vpr; v += 32) {
+    float g[NV];
+    unpack16<T>(ld_stream(dy + t * vpr + v), g);
+    uint4 raw[kMaxK];
+#pragma unroll
+    for (int k = 0; k < kMaxK; ++k)
+      if (k < K) raw[k] = ld_stream(y_perm + (int64_t)rows[k] * vpr + v);
+#pragma unroll
+    for (int k = 0; k < kMaxK; ++k) {
+      if (k < K) {
+        float f[NV], o[NV];
+        unpack16<T>(raw[k], f);
+#pragma unroll
+        for (int i = 0; i < NV; ++i) {
+          dot[k] = fmaf(g[i], f[i], dot[k]);
+          o[i] = p[k] * g[i];
+        }
+        st_stream(dy_perm + (int64_t)rows[k] * vpr + v, pack16<T>(o));
+      }
+    }
+  }
+#pragma unroll
+  for (int k = 0; k < kMaxK; ++k) {
+    if (k < K) {
+      float s = dot[k];
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
+      if (lane == 0) dprob_perm[rows[k]] = s;
+    }
+  }
+}
+
+cudaError_t launch_combine_bwd(const Ctx& c, DType dt, const void* dy, const void* y_perm, const float* prob_perm,
+                               const int32_t* row_of_slot, int64_t T, int K, int D, void* dy_perm,
+                               float* dprob_perm) {
+  if (T == 0) return cudaSuccess;
+  const int warps = 8;
+  const int vpr = (int)((int64_t)D * dsize(dt) / 16);
+  const unsigned grid = (unsigned)((T + warps - 1) / warps);
+  KernelScope ks("combine_bwd", c.stream);
+  if (dt == DType::BF16)
+    combine_bwd_kernel<bf16><<<grid, 32 * warps, 0, c.stream>>>((const uint4*)dy, (const uint4*)y_perm, prob_perm,
+                                                                row_of_slot, T, K, vpr, (uint4*)dy_perm,
+                                                                dprob_perm);
+  else
+    combine_bwd_kernel<float><<<grid, 32 * warps, 0, c.stream>>>((const uint4*)dy, (const uint4*)y_perm,
+                                                                 prob_perm, row_of_slot, T, K, vpr,
+                                                                 (uint4*)dy_perm, dprob_perm);
+  return cudaGetLastError();
+}
+
+// Dispatch backward: dx[t] = sum_k dX_perm[row_k] (fp32 accumulation);
+// dprob[t, k] = dprob_perm[row_k].
+template <typename T>
+__global__ void __launch_bounds__(256) dispatch_bwd_kernel(const uint4* __restrict__ dx_perm,
+                                                           const float* __restrict__ dprob_perm,
+                                                           const int32_t* __restrict__ row_of_slot, int64_t Tn,
+                                                           int K, int vpr, uint4* __restrict__ dx,
+                                                           float* __restrict__ dprob) {
+  constexpr int NV = Vec<T>::N;
+  const int lane = threadIdx.x & 31;
+  const int64_t t = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  if (t >= Tn) return;
+  int32_t rows[kMaxK];
+  load_rows(row_of_slot, t, K, rows);
+  if (lane < K) dprob[t * K + lane] = __ldg(dprob_perm + row_of_slot[t * K + lane]);
+  for (int v = lane; v < vpr; v += 32) {
+    float acc[NV];
+#pragma unroll
+    for (int i = 0; i < NV; ++i) acc[i] = 0.f;
+    uint4 raw[kMaxK];
+#pragma unroll
+    for (int k = 0; k < kMaxK; ++k)
+      if (k < K) raw[k] = ld_stream(dx_perm + (int64_t)rows[k] * vpr + v);
+#pragma unroll
+    for (int k = 0; k < kMaxK; ++k) {
+      if (k < K) {
+        float f[NV];
+        unpack16<T>(raw[k], f);
+#pragma unroll
+        for (int i = 0; i < NV; ++i) acc[i] += f[i];
+      }
+    }
+    st_stream(dx + t * vpr + v, pack16<T>(acc));
+  }
+}
+
+cudaError_t launch_dispatch_bwd(const Ctx& c, DType dt, const void* dx_perm, const float* dprob_perm,
+                                const int32_t* row_of_slot, int64_t T, int K, int D, void* dx, float* dprob) {
+  if (T == 0) return cudaSuccess;
+  const int warps = 8;
+  const int vpr = (int)((int64_t)D * dsize(dt) / 16);
+  const unsigned grid = (unsigned)((T + warps - 1) / warps);
+  KernelScope ks("dispatch_bwd", c.stream);
+  if (dt == DType::BF16)
+    dispatch_bwd_kernel<bf16><<<grid, 32 * warps, 0, c.stream>>>((const uint4*)dx_perm, dprob_perm, row_of_slot,
+                                                                 T, K, vpr, (uint4*)dx, dprob);
+  else
+    dispatch_bwd_kernel<float><<<grid, 32 * warps, 0, c.stream>>>((const uint4*)dx_perm, dprob_perm, row_of_slot,
+                                                                  T, K, vpr, (uint4*)dx, dprob);
+  return cudaGetLastError();
+}
+
+// w1[e, 128 i + c] = w_gate[e, 64 i + c] for c < 64, w_up[e, 64 i + c - 64] otherwise.
+__global__ void __launch_bounds__(256) pack_w1_kernel(const uint4* __restrict__ wg, const uint4* __restrict__ wu,
+                                                      int64_t rows_total, int F, int vpr, uint4* __restrict__ w1) {
+  const int64_t r = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  if (r >= rows_total) return;
+  const int lane = threadIdx.x & 31;
+  const int64_t e = r / (2 * F);
+  const int j = (int)(r % (2 * F));
+  const int blk = j / 128, c = j % 128;
+  const int f = blk * 64 + (c & 63);
+  const uint4* src = (c < 64 ? wg : wu) + (e * F + f) * vpr;
+  for (int v = lane; v < vpr; v += 32) w1[r * vpr + v] = src[v];
+}
+
+cudaError_t launch_pack_w1(const Ctx& c, DType dt, const void* w_gate, const void* w_up, int E, int F, int D,
+                           void* w1) {
+  const int64_t rows = (int64_t)E * 2 * F;
+  const int vpr = (int)((int64_t)D * dsize(dt) / 16);
+  KernelScope ks("pack_w1", c.stream);
+  pack_w1_kernel<<<(unsigned)((rows + 7) / 8), 256, 0, c.stream>>>((const uint4*)w_gate, (const uint4*)w_up, rows,
+                                                                   F, vpr, (uint4*)w1);
+  return cudaGetLastError();
+}
+
+}  // namespace moe

@@ -1,0 +1,147 @@
+"""Device buffers and the call sequence of one MoE layer step over the C ABI.
+
+PyTorch supplies device memory and the stream; every stage runs in the
+library's kernels through ``abi``.  Forward: route -> (LatentMoE down-
+projection) -> dispatch -> grouped SwiGLU experts -> combine -> (up-
+projection).  Backward runs the inverses in reverse order (Sec. 4.1 footnote:
+the three forward transfers and their three inverses).
+"""
+from __future__ import annotations
+
+import torch
+
+from . import abi
+
+
+def _dt(dtype: str):
+    return torch.bfloat16 if dtype == "bf16" else torch.float32
+
+
+class MoeLayer:
+    """All buffers of one layer step for one shape, allocated once on ``device``."""
+
+    def __init__(self, S, GBS, K, D, E, F, dtype="bf16", H=0, device="cuda"):
+        self.shape = abi.MoeShape.of(S, GBS, K, D, E, F, dtype, H)
+        self.T = T = S * GBS
+        self.TK = TK = T * K
+        self.K, self.D, self.E, self.F, self.H = K, D, E, F, H
+        self.Din = H if H else D
+        self.dtype = dtype
+        dt = _dt(dtype)
+        dev = torch.device(device)
+        f32, i32 = torch.float32, torch.int32
+        e = lambda *s, d=dt: torch.empty(*s, dtype=d, device=dev)  # noqa: E731
+        Din = self.Din
+        # weights
+        self.w_router = e(E, Din)
+        self.w1 = e(E, 2 * F, D)
+        self.w2 = e(E, D, F)
+        self.bias = None
+        self.w_down = e(D, H) if H else None
+        self.w_upp = e(H, D) if H else None
+        # forward
+        self.x = e(T, Din)
+        self.logits = e(T, E, d=f32)
+        self.topk_idx = e(T, K, d=i32)
+        self.topk_prob = e(T, K, d=f32)
+        self.x_lat = e(T, D) if H else None
+        self.expert_offsets = e(E + 1, d=i32)
+        self.row_of_slot = e(TK, d=i32)
+        self.token_of_row = e(TK, d=i32)
+        self.x_perm = e(TK, D)
+        self.prob_perm = e(TK, d=f32)
+        self.h = e(TK, 2 * F)
+        self.act = e(TK, F)
+        self.y_perm = e(TK, D)
+        self.y_lat = e(T, D) if H else None
+        self.y = e(T, Din)
+        # backward
+        self.dy = e(T, Din)
+        self.dy_lat = e(T, D) if H else None
+        self.dy_perm = e(TK, D)
+        self.dprob_perm = e(TK, d=f32)
+        self.dx_perm = e(TK, D)
+        self.dw1 = e(E, 2 * F, D, d=f32)
+        self.dw2 = e(E, D, F, d=f32)
+        self.dx_lat = e(T, D) if H else None
+        self.dprob = e(T, K, d=f32)
+        self.dx = e(T, Din)
+        self.dlogits = e(T, E, d=f32)
+        self.dw_router = e(E, Din, d=f32)
+        self.dw_down = e(D, H, d=f32) if H else None
+        self.dw_upp = e(H, D, d=f32) if H else None
+        self.ws = torch.empty(abi.moe_workspace_size(self.shape), dtype=torch.uint8, device=dev)
+
+    # ------------------------------------------------------------------
+    def load(self, inputs: dict, stream=None) -> None:
+        """Copy one ``synth.make_inputs`` dict into the device buffers and pack w1."""
+        self.x.copy_(inputs["x"], non_blocking=True)
+        self.dy.copy_(inputs["dy"], non_blocking=True)
+        self.w_router.copy_(inputs["w_router"], non_blocking=True)
+        self.w2.copy_(inputs["w2"], non_blocking=True)
+        wg = inputs["w_gate"].to(self.x.device, non_blocking=True)
+        wu = inputs["w_up"].to(self.x.device, non_blocking=True)
+        abi.moe_pack_w1(self.shape, wg, wu, self.w1, stream)
+        if self.H:
+            self.w_down.copy_(inputs["w_down"], non_blocking=True)
+            self.w_upp.copy_(inputs["w_upp"], non_blocking=True)
+        if inputs.get("bias") is not None:
+            self.bias = inputs["bias"].to(self.x.device, non_blocking=True).contiguous()
+        else:
+            self.bias = None
+
+    # ------------------------------------------------------------------
+    def forward(self, stream=None):
+        s = self.shape
+        abi.moe_route(s, self.x, self.w_router, self.bias, self.logits, self.topk_idx, self.topk_prob, self.ws,
+                      stream)
+        xd = self.x
+        if self.H:
+            abi.moe_latent_proj(s, self.H, self.D, self.x, self.w_down, self.x_lat, self.ws, stream)
+            xd = self.x_lat
+        abi.moe_dispatch(s, xd, self.topk_idx, self.topk_prob, self.expert_offsets, self.row_of_slot,
+                         self.token_of_row, self.x_perm, self.prob_perm, self.ws, stream)
+        abi.moe_expert_ffn(s, self.x_perm, self.expert_offsets, self.w1, self.w2, self.h, self.act, self.y_perm,
+                           self.ws, stream)
+        if self.H:
+            abi.moe_combine(s, self.y_perm, self.prob_perm, self.row_of_slot, self.y_lat, stream)
+            abi.moe_latent_proj(s, self.D, self.H, self.y_lat, self.w_upp, self.y, self.ws, stream)
+        else:
+            abi.moe_combine(s, self.y_perm, self.prob_perm, self.row_of_slot, self.y, stream)
+        return self.y
+
+    def backward(self, stream=None):
+        s = self.shape
+        dyd = self.dy
+        if self.H:
+            abi.moe_latent_proj_bwd(s, self.D, self.H, self.dy, self.y_lat, self.w_upp, self.dy_lat, False,
+                                    self.dw_upp, self.ws, stream)
+            dyd = self.dy_lat
+        abi.moe_combine_bwd(s, dyd, self.y_perm, self.prob_perm, self.row_of_slot, self.dy_perm, self.dprob_perm,
+                            stream)
+        abi.moe_expert_ffn_bwd(s, self.dy_perm, self.x_perm, self.h, self.act, self.expert_offsets, self.w1,
+                               self.w2, self.dx_perm, self.dw1, self.dw2, self.ws, stream)
+        if self.H:
+            abi.moe_dispatch_bwd(s, self.dx_perm, self.dprob_perm, self.row_of_slot, self.dx_lat, self.dprob, stream)
+            abi.moe_latent_proj_bwd(s, self.H, self.D, self.dx_lat, self.x, self.w_down, self.dx, False,
+                                    self.dw_down, self.ws, stream)
+        else:
+            abi.moe_dispatch_bwd(s, self.dx_perm, self.dprob_perm, self.row_of_slot, self.dx, self.dprob, stream)
+        abi.moe_route_bwd(s, self.x, self.w_router, self.topk_idx, self.topk_prob, self.dprob, self.dx,
+                          self.dw_router, self.dlogits, self.ws, stream)
+        return self.dx
+
+    def step(self, stream=None):
+        self.forward(stream)
+        self.backward(stream)
+
+    # ------------------------------------------------------------------
+    def unpack_w1_like(self, t: torch.Tensor):
+        """Split a packed [E, 2F, D] tensor (w1 or dw1) into gate and up [E, F, D]."""
+        v = t.view(self.E, self.F // 64, 2, 64, self.D)
+        return v[:, :, 0].reshape(self.E, self.F, self.D), v[:, :, 1].reshape(self.E, self.F, self.D)
+
+    def unpack_h(self, h: torch.Tensor):
+        """Split a packed [rows, 2F] tensor (h or dH) into its gate and up halves [rows, F]."""
+        v = h.view(h.shape[0], self.F // 64, 2, 64)
+        return v[:, :, 0].reshape(h.shape[0], self.F), v[:, :, 1].reshape(h.shape[0], self.F)

@@ -1,0 +1,50 @@
+"""Helpers shared by the GPU parity tests."""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+import oracle as O
+import synth
+
+# Tolerances of the layer (float outputs and gradients: relative Frobenius
+# error against the float64 oracle; routed probabilities: absolute error).
+REL_FROB = 1e-2
+PROB_ABS = 1e-5
+LOGIT_REL = 1e-5
+
+
+def rel_frob(a, b) -> float:
+    a = np.asarray(a, dtype=np.float64)
+    b = np.asarray(b, dtype=np.float64)
+    den = np.linalg.norm(b)
+    if den == 0.0:
+        return float(np.linalg.norm(a))
+    return float(np.linalg.norm(a - b) / den)
+
+
+def f64(t) -> np.ndarray:
+    return t.detach().float().cpu().double().numpy() if t.dtype == torch.bfloat16 else \
+        t.detach().cpu().double().numpy()
+
+
+def i64(t) -> np.ndarray:
+    return t.detach().cpu().numpy().astype(np.int64)
+
+
+def make_layer(w: synth.Workload, T: int | None = None, seed: int | None = None, inputs: dict | None = None):
+    """Build a MoeLayer for workload ``w`` (token count T), load seeded inputs, run forward+backward."""
+    from paper_2608_28511_gb300.layer import MoeLayer
+    T = w.T if T is None else T
+    if inputs is None:
+        inputs = synth.make_inputs(w, seed=seed, T=T)
+    layer = MoeLayer(T, 1, w.K, w.D, w.E, w.F, w.dtype, w.H)
+    layer.load(inputs)
+    layer.forward()
+    layer.backward()
+    torch.cuda.synchronize()
+    return layer, inputs
+
+
+def oracle_inputs(inputs: dict) -> dict:
+    return {k: synth.to_f64(v) for k, v in inputs.items()}

@@ -1,0 +1,260 @@
+"""GPU parity of every stage of the layer against the float64 oracle.
+
+Stage-isolated checks feed the oracle the GPU's own inputs to that stage, so
+index work is compared bit for bit and float work within the layer's
+tolerances (relative Frobenius 1e-2, probabilities 1e-5 absolute, logits
+1e-5 relative).  End-to-end checks run the oracle from the raw inputs.
+Sizes span several GEMM tiles with ragged tails and finish in seconds.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+import synth
+from tests.gpu_util import LOGIT_REL, PROB_ABS, REL_FROB, f64, i64, make_layer, oracle_inputs, rel_frob
+
+pytestmark = pytest.mark.gpu
+
+W = synth.Workload
+CASES = {
+    "tiny_fp32": synth.TINY,
+    "mid_bf16": W("mid_bf16", S=500, GBS=2, D=256, E=16, K=4, F=320),
+    "mid_skew": W("mid_skew", S=350, GBS=2, D=256, E=16, K=4, F=256, skew_bias=True),
+    "mid_latent": W("mid_latent", S=300, GBS=2, D=256, E=32, K=4, F=192, H=512),
+    "mid_fp32": W("mid_fp32", S=300, GBS=1, D=192, E=12, K=3, F=192, dtype="f32"),
+    "wide_bf16": W("wide_bf16", S=384, GBS=1, D=1024, E=8, K=2, F=768),
+}
+
+_cache = {}
+
+
+def run(name):
+    if name not in _cache:
+        w = CASES[name]
+        layer, inputs = make_layer(w)
+        _cache[name] = (w, layer, inputs, oracle_inputs(inputs))
+    return _cache[name]
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    import __graft_entry__
+    __graft_entry__.build()
+    yield
+    _cache.clear()
+
+
+names = list(CASES)
+
+
+@pytest.mark.parametrize("name", names)
+def test_route_stage(name):
+    w, L, inp, o = run(name)
+    z_ref = O.router_logits(o["x"], o["w_router"], o["bias"])
+    z_gpu = f64(L.logits)
+    assert rel_frob(z_gpu, z_ref) <= LOGIT_REL
+    idx_ref, prob_ref = O.top_k_route(z_gpu, w.K)           # stage-isolated: the GPU's logits
+    assert (i64(L.topk_idx) == idx_ref).all()
+    assert np.abs(f64(L.topk_prob) - prob_ref).max() <= PROB_ABS
+    assert np.abs(f64(L.topk_prob).sum(axis=1) - 1.0).max() <= 1e-6
+
+
+@pytest.mark.parametrize("name", names)
+def test_permutation_stage(name):
+    w, L, inp, o = run(name)
+    idx = i64(L.topk_idx)
+    off, ros, tor = O.expert_permutation(idx, w.E)
+    assert (i64(L.expert_offsets) == off).all()
+    assert (i64(L.row_of_slot) == ros).all()
+    assert (i64(L.token_of_row) == tor).all()
+    x_disp = L.x_lat if w.H else L.x
+    assert torch.equal(L.x_perm, x_disp[L.token_of_row.long()])
+    assert torch.equal(L.prob_perm[L.row_of_slot.long()], L.topk_prob.reshape(-1))
+    # Eq. 1 payload of the forward dispatch (I7)
+    assert L.x_perm.numel() * L.x_perm.element_size() + L.prob_perm.numel() * 4 == w.T * w.K * (w.D * w.b_x + 4)
+
+
+@pytest.mark.parametrize("name", names)
+def test_expert_ffn_stage(name):
+    w, L, inp, o = run(name)
+    g, u, a, y = O.expert_ffn(f64(L.x_perm), i64(L.expert_offsets), o["w_gate"], o["w_up"], o["w2"])
+    hg, hu = L.unpack_h(L.h)
+    assert rel_frob(f64(hg), g) <= REL_FROB
+    assert rel_frob(f64(hu), u) <= REL_FROB
+    assert rel_frob(f64(L.act), a) <= REL_FROB
+    assert rel_frob(f64(L.y_perm), y) <= REL_FROB
+
+
+@pytest.mark.parametrize("name", names)
+def test_combine_stage(name):
+    w, L, inp, o = run(name)
+    y = O.combine(f64(L.y_perm), f64(L.prob_perm), i64(L.row_of_slot), w.T, w.K)
+    y_gpu = L.y_lat if w.H else L.y
+    assert rel_frob(f64(y_gpu), y) <= REL_FROB
+    if w.H:
+        assert rel_frob(f64(L.y), O.latent_project(f64(L.y_lat), o["w_upp"])) <= REL_FROB
+        assert rel_frob(f64(L.x_lat), O.latent_project(o["x"], o["w_down"])) <= REL_FROB
+
+
+@pytest.mark.parametrize("name", names)
+def test_combine_bwd_stage(name):
+    w, L, inp, o = run(name)
+    dy = f64(L.dy_lat) if w.H else o["dy"]
+    dyp, dpp = O.combine_bwd(dy, f64(L.y_perm), f64(L.prob_perm), i64(L.token_of_row))
+    assert rel_frob(f64(L.dy_perm), dyp) <= REL_FROB
+    assert rel_frob(f64(L.dprob_perm), dpp) <= REL_FROB
+    if w.H:
+        dyl, dwu = O.latent_project_bwd(o["dy"], f64(L.y_lat), o["w_upp"])
+        assert rel_frob(f64(L.dy_lat), dyl) <= REL_FROB
+        assert rel_frob(f64(L.dw_upp), dwu) <= REL_FROB
+
+
+@pytest.mark.parametrize("name", names)
+def test_expert_ffn_bwd_stage(name):
+    w, L, inp, o = run(name)
+    hg, hu = L.unpack_h(L.h)
+    dxp, dwg, dwu, dw2 = O.expert_ffn_bwd(f64(L.dy_perm), f64(L.x_perm), f64(hg), f64(hu), i64(L.expert_offsets),
+                                          o["w_gate"], o["w_up"], o["w2"])
+    gg, gu = L.unpack_w1_like(L.dw1)
+    assert rel_frob(f64(L.dx_perm), dxp) <= REL_FROB
+    assert rel_frob(f64(gg), dwg) <= REL_FROB
+    assert rel_frob(f64(gu), dwu) <= REL_FROB
+    assert rel_frob(f64(L.dw2), dw2) <= REL_FROB
+    # experts with no rows get exactly zero weight gradients
+    cnt = np.diff(i64(L.expert_offsets))
+    for e in np.nonzero(cnt == 0)[0]:
+        assert float(L.dw1[e].abs().max()) == 0.0 and float(L.dw2[e].abs().max()) == 0.0
+
+
+@pytest.mark.parametrize("name", names)
+def test_dispatch_and_route_bwd_stage(name):
+    w, L, inp, o = run(name)
+    dx_e, dprob = O.dispatch_bwd(f64(L.dx_perm), f64(L.dprob_perm), i64(L.row_of_slot), w.T, w.K)
+    assert np.array_equal(f64(L.dprob), dprob)                     # a pure gather of fp32 values
+    dz, dx_r, dw_r = O.route_bwd(o["x"], o["w_router"], i64(L.topk_idx), f64(L.topk_prob), f64(L.dprob))
+    assert rel_frob(f64(L.dlogits), dz) <= REL_FROB
+    assert rel_frob(f64(L.dw_router), dw_r) <= REL_FROB
+    if w.H:
+        assert rel_frob(f64(L.dx_lat), dx_e) <= REL_FROB
+        dx_h, dw_down = O.latent_project_bwd(f64(L.dx_lat), o["x"], o["w_down"])
+        assert rel_frob(f64(L.dw_down), dw_down) <= REL_FROB
+        assert rel_frob(f64(L.dx), dx_h + dx_r) <= REL_FROB
+    else:
+        assert rel_frob(f64(L.dx), dx_e + dx_r) <= REL_FROB
+    # I5: dz rows sum to zero
+    assert np.abs(f64(L.dlogits).sum(axis=1)).max() <= 1e-5 * max(1.0, np.abs(dz).max())
+
+
+@pytest.mark.parametrize("name", names)
+def test_end_to_end(name):
+    w, L, inp, o = run(name)
+    z = O.router_logits(o["x"], o["w_router"], o["bias"])
+    idx_own, _ = O.top_k_route(z, w.K)
+    idx_gpu = i64(L.topk_idx)
+    ties = set(O.near_tie_tokens(z, w.K).tolist())
+    differ = set(np.nonzero((idx_own != idx_gpu).any(axis=1))[0].tolist())
+    assert differ <= ties, f"routing differs outside near-ties: {sorted(differ - ties)[:10]}"
+    kw = dict(w_down=o.get("w_down"), w_upp=o.get("w_upp"))
+    fwd = O.layer_forward(o["x"], o["w_router"], o["w_gate"], o["w_up"], o["w2"], w.K, bias=o["bias"],
+                          idx_override=idx_gpu, **kw)
+    bwd = O.layer_backward(fwd, o["dy"], o["x"], o["w_router"], o["w_gate"], o["w_up"], o["w2"], **kw)
+    assert np.abs(f64(L.topk_prob) - fwd["prob"]).max() <= PROB_ABS
+    assert rel_frob(f64(L.y), fwd["y"]) <= REL_FROB
+    assert rel_frob(f64(L.dx), bwd["dx"]) <= REL_FROB
+    gg, gu = L.unpack_w1_like(L.dw1)
+    assert rel_frob(f64(gg), bwd["dw_gate"]) <= REL_FROB
+    assert rel_frob(f64(gu), bwd["dw_up"]) <= REL_FROB
+    assert rel_frob(f64(L.dw2), bwd["dw2"]) <= REL_FROB
+    assert rel_frob(f64(L.dw_router), bwd["dw_router"]) <= REL_FROB
+    assert rel_frob(f64(L.dlogits), bwd["dz"]) <= REL_FROB
+    assert rel_frob(f64(L.dprob), bwd["dprob"]) <= REL_FROB
+    if w.H:
+        assert rel_frob(f64(L.dw_down), bwd["dw_down"]) <= REL_FROB
+        assert rel_frob(f64(L.dw_upp), bwd["dw_upp"]) <= REL_FROB
+
+
+# ---------------------------------------------------------------------------
+# Edge cases
+# ---------------------------------------------------------------------------
+
+EDGE = [
+    W("t1", S=1, GBS=1, D=128, E=8, K=2, F=128),
+    W("t3", S=3, GBS=1, D=128, E=8, K=2, F=128),
+    W("t127", S=127, GBS=1, D=128, E=8, K=2, F=128),
+    W("e_eq_k", S=64, GBS=1, D=128, E=4, K=4, F=128),
+    W("k1", S=200, GBS=1, D=128, E=8, K=1, F=192),
+    W("t3_fp32", S=3, GBS=1, D=64, E=4, K=2, F=64, dtype="f32"),
+    W("k16", S=50, GBS=1, D=64, E=32, K=16, F=64),
+]
+
+
+@pytest.mark.parametrize("w", EDGE, ids=[e.name for e in EDGE])
+def test_edge_shapes_end_to_end(w):
+    L, inp = make_layer(w)
+    o = oracle_inputs(inp)
+    idx_gpu = i64(L.topk_idx)
+    off, ros, tor = O.expert_permutation(idx_gpu, w.E)
+    assert (i64(L.expert_offsets) == off).all() and (i64(L.row_of_slot) == ros).all()
+    fwd = O.layer_forward(o["x"], o["w_router"], o["w_gate"], o["w_up"], o["w2"], w.K, idx_override=idx_gpu)
+    bwd = O.layer_backward(fwd, o["dy"], o["x"], o["w_router"], o["w_gate"], o["w_up"], o["w2"])
+    assert rel_frob(f64(L.y), fwd["y"]) <= REL_FROB
+    assert rel_frob(f64(L.dx), bwd["dx"]) <= REL_FROB
+    assert rel_frob(f64(L.dw2), bwd["dw2"]) <= REL_FROB
+    gg, gu = L.unpack_w1_like(L.dw1)
+    assert rel_frob(f64(gg), bwd["dw_gate"]) <= REL_FROB
+    assert rel_frob(f64(L.dw_router), bwd["dw_router"]) <= REL_FROB
+
+
+def test_all_tokens_on_one_expert():
+    w = W("one_expert", S=300, GBS=1, D=128, E=8, K=1, F=128)
+    inp = synth.make_inputs(w)
+    inp["bias"] = torch.zeros(8)
+    inp["bias"][5] = 1000.0
+    L, _ = make_layer(w, inputs=inp)
+    off = i64(L.expert_offsets)
+    assert off.tolist() == [0, 0, 0, 0, 0, 0, 300, 300, 300]
+    assert (i64(L.token_of_row) == np.arange(300)).all()
+    o = oracle_inputs(inp)
+    fwd = O.layer_forward(o["x"], o["w_router"], o["w_gate"], o["w_up"], o["w2"], 1, bias=o["bias"])
+    assert rel_frob(f64(L.y), fwd["y"]) <= REL_FROB
+    for e in (0, 1, 7):
+        assert float(L.dw2[e].abs().max()) == 0.0
+
+
+def test_deterministic_bitwise():
+    w = CASES["mid_bf16"]
+    inp = synth.make_inputs(w)
+    L1, _ = make_layer(w, inputs=inp)
+    L2, _ = make_layer(w, inputs=inp)
+    for name in ("logits", "topk_idx", "topk_prob", "expert_offsets", "row_of_slot", "token_of_row", "x_perm",
+                 "h", "act", "y_perm", "y", "dy_perm", "dprob_perm", "dx_perm", "dw1", "dw2", "dx", "dlogits",
+                 "dw_router"):
+        a, b = getattr(L1, name), getattr(L2, name)
+        assert torch.equal(a.view(torch.uint8) if a.dtype != torch.bfloat16 else a.view(torch.int16),
+                           b.view(torch.uint8) if b.dtype != torch.bfloat16 else b.view(torch.int16)), name
+
+
+def test_out_of_range_expert_index_sets_status_word():
+    from paper_2608_28511_gb300 import abi
+    w = W("badidx", S=64, GBS=1, D=128, E=8, K=2, F=128)
+    shp = abi.MoeShape.from_workload(w)
+    dev = "cuda"
+    idx = torch.randint(0, 8, (64, 2), dtype=torch.int32, device=dev)
+    idx[:, 1] = (idx[:, 0] + 1) % 8
+    idx[7, 1] = 9            # out of range
+    idx[9, 0] = -3           # out of range
+    prob = torch.full((64, 2), 0.5, device=dev)
+    x = torch.randn(64, 128, device=dev).to(torch.bfloat16)
+    off = torch.empty(9, dtype=torch.int32, device=dev)
+    ros = torch.empty(128, dtype=torch.int32, device=dev)
+    tor = torch.empty(128, dtype=torch.int32, device=dev)
+    xp = torch.empty(128, 128, dtype=torch.bfloat16, device=dev)
+    pp = torch.empty(128, device=dev)
+    ws = torch.empty(abi.moe_workspace_size(shp), dtype=torch.uint8, device=dev)
+    assert abi.moe_check_device_status() == 0
+    abi.moe_dispatch(shp, x, idx, prob, off, ros, tor, xp, pp, ws)
+    assert abi.moe_device_status_word() & 1
+    assert abi.moe_check_device_status() == -7
+    assert abi.moe_check_device_status() == 0      # cleared
+    assert int(off[-1]) == 126                     # only valid slots are counted
