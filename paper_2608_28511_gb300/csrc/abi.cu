@@ -484,6 +484,7 @@ int moe_expert_ffn_bwd(const moe_shape_t* shape, const void* dy_perm, const void
   b.b_type = d.dt;
   b.sb_n = 1;
   b.sb_k = d.F;
+  b.max_rows = d.TK;
   b.C = dw2;
   b.c_type = DType::F32;
   b.ldc = d.F;
@@ -525,6 +526,7 @@ int moe_expert_ffn_bwd(const moe_shape_t* shape, const void* dy_perm, const void
   w.b_type = d.dt;
   w.sb_n = 1;
   w.sb_k = d.D;
+  w.max_rows = d.TK;
   w.C = dw1;
   w.c_type = DType::F32;
   w.ldc = d.D;

@@ -1,10 +1,182 @@
-// Tensor-core grouped GEMM engine (placeholder until the tcgen05 path lands).
-#include "launch.h"
+// Host side of the tcgen05 engine: which GemmDesc shapes it takes, tensor-map
+// encoding (cuTensorMapEncodeTiled through the runtime's driver entry point)
+// and the launch of the matching kernel instantiation.
+#include <cstring>
+#include <mutex>
+
+#include "gemm_tc.cuh"
 
 namespace moe {
 
-bool gemm_tc_supports(const GemmDesc&) { return false; }
+using tc::BM;
+using tc::Cfg;
+using tc::Params;
 
-cudaError_t launch_gemm_tc(const Ctx&, const GemmDesc&, const char*) { return cudaErrorNotSupported; }
+namespace {
+
+using EncodeFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                              const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                              CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeFn encode_fn() {
+  static EncodeFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeFn>(ptr);
+  });
+  return fn;
+}
+
+// 2-D bf16 tensor map: `inner` contiguous elements per row, `outer` rows of
+// `stride_bytes`, box {box_inner, box_outer}, 128-byte swizzle, zero fill.
+bool make_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer, uint64_t stride_bytes,
+              uint32_t box_inner, uint32_t box_outer) {
+  EncodeFn fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {inner, outer};
+  cuuint64_t strides[1] = {stride_bytes};
+  cuuint32_t box[2] = {box_inner, box_outer};
+  cuuint32_t es[2] = {1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+bool al16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+
+struct Plan {
+  int bn;
+  bool a_mn, b_mn;
+  int64_t lda, ldb;
+};
+
+bool make_plan(const GemmDesc& d, Plan* pl) {
+  if (d.a_type != DType::BF16 || d.b_type != DType::BF16) return false;
+  if (d.N <= 0 || (d.group != Group::M && d.M <= 0) || (d.group != Group::K && d.K <= 0)) return false;
+  if (d.sa_k == 1 && d.sa_m > 1) { pl->a_mn = false; pl->lda = d.sa_m; }
+  else if (d.sa_m == 1 && d.sa_k > 1) { pl->a_mn = true; pl->lda = d.sa_k; }
+  else return false;
+  if (d.sb_k == 1 && d.sb_n > 1) { pl->b_mn = false; pl->ldb = d.sb_n; }
+  else if (d.sb_n == 1 && d.sb_k > 1) { pl->b_mn = true; pl->ldb = d.sb_k; }
+  else return false;
+  if ((pl->lda * 2) % 16 || (pl->ldb * 2) % 16) return false;
+  if (!al16(d.A) || !al16(d.B) || !al16(d.C)) return false;
+  if (d.group == Group::K && !(pl->a_mn && pl->b_mn)) return false;
+  if (d.group == Group::M && pl->a_mn) return false;
+  if (d.group == Group::M && (d.sb_g % pl->ldb)) return false;
+  if (d.group != Group::Dense && (d.num_groups <= 0 || d.num_groups > kMaxE || !d.offsets)) return false;
+  const size_t cs = dsize(d.c_type);
+  if ((d.ldc * cs) % 16) return false;
+  switch (d.epi) {
+    case Epi::Store: break;
+    case Epi::StoreBias: if (d.c_type != DType::F32) return false; break;
+    case Epi::Accum: if (d.c_type != DType::BF16) return false; break;
+    case Epi::SwigluFwd:
+      if (d.c_type != DType::BF16 || d.N % 128 || !d.aux || !al16(d.aux)) return false;
+      break;
+    case Epi::SwigluBwd:
+      if (d.c_type != DType::BF16 || d.N % 64 || !d.h_in || !al16(d.h_in)) return false;
+      break;
+  }
+  pl->bn = 256;
+  if (d.group == Group::Dense && d.epi == Epi::StoreBias) pl->bn = d.N <= 64 ? 64 : (d.N <= 128 ? 128 : 256);
+  return true;
+}
+
+template <int BN, bool A_MN, bool B_MN, int GROUP, int EPI, typename TC>
+cudaError_t launch_inst(const Ctx& c, const Params& p, int grid) {
+  auto k = tc::gemm_tc_kernel<BN, A_MN, B_MN, GROUP, EPI, TC>;
+  static bool configured = false;
+  if (!configured) {
+    cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg<BN>::kSmem);
+    if (e != cudaSuccess) return e;
+    configured = true;
+  }
+  k<<<grid, tc::kThreads, Cfg<BN>::kSmem, c.stream>>>(p);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+bool gemm_tc_supports(const GemmDesc& d) {
+  Plan pl;
+  if (!make_plan(d, &pl)) return false;
+  const int g = (int)d.group, e = (int)d.epi;
+  const bool f32 = d.c_type == DType::F32;
+  // the instantiated combinations
+  if (g == 1 && !pl.a_mn && !pl.b_mn && e == 3 && !f32) return true;
+  if (g == 1 && !pl.a_mn && !pl.b_mn && e == 0 && !f32) return true;
+  if (g == 1 && !pl.a_mn && pl.b_mn && e == 4 && !f32) return true;
+  if (g == 1 && !pl.a_mn && pl.b_mn && e == 0 && !f32) return true;
+  if (g == 2 && pl.a_mn && pl.b_mn && e == 0 && f32) return true;
+  if (g == 0 && !pl.a_mn && !pl.b_mn && e == 1 && f32) return true;
+  if (g == 0 && !pl.a_mn && !pl.b_mn && e == 0 && !f32) return true;
+  if (g == 0 && !pl.a_mn && pl.b_mn && (e == 0 || e == 2) && !f32) return true;
+  if (g == 0 && pl.a_mn && pl.b_mn && e == 0 && f32) return true;
+  return false;
+}
+
+cudaError_t launch_gemm_tc(const Ctx& c, const GemmDesc& d, const char* name) {
+  Plan pl;
+  if (!make_plan(d, &pl) || !gemm_tc_supports(d)) return cudaErrorNotSupported;
+  Params p;
+  memset(&p, 0, sizeof(p));
+  const int bn = pl.bn;
+  // A: K-major box {64 k, 128 m}; MN-major box {64 m, 64 k}
+  const int64_t a_rows = pl.a_mn ? (d.group == Group::K ? d.max_rows : d.K) : (d.group == Group::M ? d.max_rows : d.M);
+  const int64_t a_inner = pl.a_mn ? d.M : d.K;
+  if (!make_map(&p.ta, d.A, a_inner, a_rows, pl.lda * 2, 64, pl.a_mn ? 64 : BM)) return cudaErrorInvalidValue;
+  // B: K-major box {64 k, BN n}; MN-major box {64 n, 64 k}
+  const int64_t grows = d.group == Group::M ? d.sb_g / pl.ldb : 0;
+  int64_t b_rows;
+  if (pl.b_mn) b_rows = d.group == Group::M ? grows * d.num_groups : (d.group == Group::K ? d.max_rows : d.K);
+  else b_rows = d.group == Group::M ? grows * d.num_groups : d.N;
+  const int64_t b_inner = pl.b_mn ? d.N : d.K;
+  if (!make_map(&p.tb, d.B, b_inner, b_rows, pl.ldb * 2, 64, pl.b_mn ? 64 : bn)) return cudaErrorInvalidValue;
+  p.M = d.M;
+  p.N = d.N;
+  p.K = d.K;
+  p.b_group_rows = grows;
+  p.num_groups = d.group == Group::Dense ? 1 : d.num_groups;
+  p.tiles_m = (int)((d.M + BM - 1) / BM);
+  p.tiles_n = (int)((d.N + bn - 1) / bn);
+  p.offsets = d.offsets;
+  p.C = d.C;
+  p.ldc = d.ldc;
+  p.sc_g = d.sc_g;
+  p.bias = d.bias;
+  p.h_in = d.h_in;
+  p.aux = d.aux;
+  p.err = c.err;
+  int64_t ub;
+  if (d.group == Group::Dense) ub = (int64_t)p.tiles_m * p.tiles_n;
+  else if (d.group == Group::M) ub = ((d.max_rows + BM - 1) / BM + d.num_groups) * p.tiles_n;
+  else ub = (int64_t)d.num_groups * p.tiles_m * p.tiles_n;
+  if (ub <= 0) return cudaSuccess;
+  const int grid = (int)(ub < c.num_sms ? ub : c.num_sms);
+  const int g = (int)d.group, e = (int)d.epi;
+  const bool f32 = d.c_type == DType::F32;
+  KernelScope ks(name, c.stream);
+  if (g == 1 && !pl.b_mn && e == 3) return launch_inst<256, false, false, 1, 3, bf16>(c, p, grid);
+  if (g == 1 && !pl.b_mn && e == 0) return launch_inst<256, false, false, 1, 0, bf16>(c, p, grid);
+  if (g == 1 && pl.b_mn && e == 4) return launch_inst<256, false, true, 1, 4, bf16>(c, p, grid);
+  if (g == 1 && pl.b_mn && e == 0) return launch_inst<256, false, true, 1, 0, bf16>(c, p, grid);
+  if (g == 2) return launch_inst<256, true, true, 2, 0, float>(c, p, grid);
+  if (g == 0 && e == 1) {
+    if (bn == 64) return launch_inst<64, false, false, 0, 1, float>(c, p, grid);
+    if (bn == 128) return launch_inst<128, false, false, 0, 1, float>(c, p, grid);
+    return launch_inst<256, false, false, 0, 1, float>(c, p, grid);
+  }
+  if (g == 0 && !pl.a_mn && !pl.b_mn && e == 0) return launch_inst<256, false, false, 0, 0, bf16>(c, p, grid);
+  if (g == 0 && !pl.a_mn && pl.b_mn && e == 0) return launch_inst<256, false, true, 0, 0, bf16>(c, p, grid);
+  if (g == 0 && !pl.a_mn && pl.b_mn && e == 2) return launch_inst<256, false, true, 0, 2, bf16>(c, p, grid);
+  if (g == 0 && pl.a_mn && pl.b_mn && f32) return launch_inst<256, true, true, 0, 0, float>(c, p, grid);
+  return cudaErrorNotSupported;
+}
 
 }  // namespace moe

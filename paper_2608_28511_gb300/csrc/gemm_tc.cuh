@@ -1,0 +1,564 @@
+// Tensor-core grouped GEMM engine for sm_103a: TMA -> shared memory ->
+// tcgen05.mma (bf16 x bf16 -> fp32 in TMEM) -> tcgen05.ld -> fused epilogue.
+//
+// C(m, n) = sum_k A(m, k) B(n, k) over 128 x BN x 64 tiles.  One persistent
+// CTA per SM walks a static tile sequence decoded on the device from the
+// expert offsets (no host synchronisation).  Warp roles (192 threads):
+//   warp 0      TMA producer (one lane) filling a kStages-deep smem ring;
+//   warp 1      TMEM allocator and MMA issuer (one lane issues, all wait);
+//   warps 2..5  epilogue: TMEM -> registers -> global, one accumulator row
+//               per thread, double-buffered accumulators (2 x BN columns).
+// Operands are staged with 128-byte swizzle; A and B may each be K-major
+// (rows of K contiguous) or MN-major (rows of M / N contiguous).
+//
+// Grouping: Group::M tiles never mix experts in an output row range (rows
+// past an expert's end are computed and dropped); Group::K reduces each
+// expert over its own row range, zeroing the rows of the last partial k-block
+// that belong to the next expert before the MMA reads them.
+//
+// Every mbarrier wait is bounded (kWaitLimitNs); on expiry the CTA sets the
+// device status word, drains its own copies and MMAs, frees TMEM and exits.
+#pragma once
+
+#include <cuda.h>
+
+#include "common.cuh"
+#include "launch.h"
+
+namespace moe {
+namespace tc {
+
+constexpr int BM = 128;
+constexpr int BK = 64;                  // bf16: 128 bytes, one swizzle row
+constexpr int kThreads = 192;
+constexpr uint64_t kWaitLimitNs = 4000000000ull;
+
+struct Params {
+  CUtensorMap ta;
+  CUtensorMap tb;
+  int64_t M, N, K;
+  int64_t b_group_rows;   // rows of B's tensor map per group (Group::M)
+  int num_groups;
+  int tiles_m, tiles_n;
+  const int32_t* offsets;
+  void* C;
+  int64_t ldc, sc_g;
+  const float* bias;
+  const void* h_in;
+  void* aux;
+  uint32_t* err;
+};
+
+// ---------------------------------------------------------------------------
+// PTX wrappers
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}\n"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+__device__ __forceinline__ uint64_t global_timer_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+// Wait for phase `parity` of `bar`; false if the CTA aborted or the limit expired.
+__device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, volatile int* abort_flag,
+                                             uint32_t* err) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = global_timer_ns();
+  for (uint32_t i = 1;; ++i) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((i & 63u) == 0) {
+      if (*abort_flag) return false;
+      if (global_timer_ns() - t0 > kWaitLimitNs) {
+        *abort_flag = 1;
+        set_error(err, kErrTimeout);
+        return false;
+      }
+    }
+  }
+}
+// Same, ignoring the abort flag (used while draining).
+__device__ __forceinline__ bool wait_drain(uint32_t bar, uint32_t parity, uint64_t limit_ns) {
+  const uint64_t t0 = global_timer_ns();
+  while (!mbar_try_wait(bar, parity)) {
+    if (global_timer_ns() - t0 > limit_ns) return false;
+  }
+  return true;
+}
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, uint32_t bar, int x, int y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4}], [%2];" ::
+          "r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(x), "r"(y)
+      : "memory");
+}
+__device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap* map) {
+  asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
+}
+__device__ __forceinline__ void tmem_alloc(uint32_t dst_smem, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem), "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish() {
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+__device__ __forceinline__ void fence_barrier_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                         uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}\n" ::"r"(d_tmem),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+__device__ __forceinline__ void mma_commit(uint32_t bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+               : "memory");
+}
+// 32 consecutive fp32 columns of this warp's 32 TMEM lanes (one row per thread).
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+      "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+        "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+        "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+  // the registers are tied to the wait so no use is scheduled before it
+  asm volatile("tcgen05.wait::ld.sync.aligned;"
+               : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]), "+r"(r[7]),
+                 "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]), "+r"(r[14]),
+                 "+r"(r[15]), "+r"(r[16]), "+r"(r[17]), "+r"(r[18]), "+r"(r[19]), "+r"(r[20]), "+r"(r[21]),
+                 "+r"(r[22]), "+r"(r[23]), "+r"(r[24]), "+r"(r[25]), "+r"(r[26]), "+r"(r[27]), "+r"(r[28]),
+                 "+r"(r[29]), "+r"(r[30]), "+r"(r[31])
+               :
+               : "memory");
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// Shared-memory matrix descriptor, 128-byte swizzle, tcgen05 version bits.
+//  K-major : LBO unused, SBO = 1024 (8 rows x 128 B); a 16-element k step is +32 B.
+//  MN-major: LBO = byte stride between 64-element MN chunks, SBO = 1024
+//            (8 k rows x 128 B); a 16-element k step is +2048 B.
+__device__ __forceinline__ uint64_t make_sdesc(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);
+  d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;
+  d |= (uint64_t)((sbo >> 4) & 0x3FFFu) << 32;
+  d |= (uint64_t)1 << 46;
+  d |= (uint64_t)2 << 61;
+  return d;
+}
+
+// Instruction descriptor for kind::f16: fp32 accumulator, bf16 A and B,
+// operand majorness, N >> 3 at bit 17, M >> 4 at bit 24.
+__host__ __device__ constexpr uint32_t make_idesc(int bn, bool a_mn, bool b_mn) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((a_mn ? 1u : 0u) << 15) | ((b_mn ? 1u : 0u) << 16) |
+         ((uint32_t)(bn >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
+}
+
+template <int BN>
+struct Cfg {
+  static constexpr int kABytes = BM * BK * 2;
+  static constexpr int kBBytes = BN * BK * 2;
+  static constexpr int kStageBytes = kABytes + kBBytes;
+  static constexpr int kStages = (196608 / kStageBytes) < 8 ? (196608 / kStageBytes) : 8;
+  static constexpr int kCols = 2 * BN;  // double-buffered fp32 accumulator
+  static constexpr int kSmem = kStages * kStageBytes + 1024 /*align*/ + 512 /*barriers*/;
+};
+
+struct Tile {
+  int g;
+  int64_t row0, row_end, n0, kbeg, kend;
+  int nkb;
+};
+
+// Tile t of the static sequence.  GROUP: 0 dense, 1 by M, 2 by K.
+template <int GROUP>
+__device__ __forceinline__ void decode_tile(const Params& p, int t, const int* s_off, const int* s_pref,
+                                            Tile& ti) {
+  if (GROUP == 0) {
+    const int mt = t / p.tiles_n, nt = t % p.tiles_n;
+    ti.g = 0;
+    ti.row0 = (int64_t)mt * BM;
+    ti.row_end = p.M;
+    ti.n0 = nt;
+    ti.kbeg = 0;
+    ti.kend = p.K;
+  } else if (GROUP == 1) {
+    const int mb = t / p.tiles_n, nt = t % p.tiles_n;
+    int lo = 0, hi = p.num_groups - 1;  // last g with s_pref[g] <= mb
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (s_pref[mid] <= mb) lo = mid;
+      else hi = mid - 1;
+    }
+    ti.g = lo;
+    ti.row0 = (int64_t)s_off[lo] + (int64_t)(mb - s_pref[lo]) * BM;
+    ti.row_end = s_off[lo + 1];
+    ti.n0 = nt;
+    ti.kbeg = 0;
+    ti.kend = p.K;
+  } else {
+    const int per = p.tiles_m * p.tiles_n;
+    const int g = t / per, rem = t % per;
+    ti.g = g;
+    ti.row0 = (int64_t)(rem / p.tiles_n) * BM;
+    ti.row_end = p.M;
+    ti.n0 = rem % p.tiles_n;
+    ti.kbeg = s_off[g];
+    ti.kend = s_off[g + 1];
+  }
+  ti.nkb = (int)((ti.kend - ti.kbeg + BK - 1) / BK);
+}
+
+__device__ __forceinline__ int64_t imin64(int64_t a, int64_t b) { return a < b ? a : b; }
+
+__device__ __forceinline__ float silu_f(float v) { return v / (1.0f + __expf(-v)); }
+__device__ __forceinline__ float sigmoid_f(float v) { return 1.0f / (1.0f + __expf(-v)); }
+
+template <typename T>
+__device__ __forceinline__ void store_row32(T* dst, const float* v, int valid) {
+  constexpr int NV = Vec<T>::N;
+  if (valid >= 32) {
+#pragma unroll
+    for (int i = 0; i < 32; i += NV) *reinterpret_cast<uint4*>(dst + i) = pack16<T>(v + i);
+  } else {
+#pragma unroll
+    for (int i = 0; i < 32; ++i)
+      if (i < valid) dst[i] = from_f32<T>(v[i]);
+  }
+}
+template <typename T>
+__device__ __forceinline__ void load_row32(const T* src, float* v) {
+  constexpr int NV = Vec<T>::N;
+#pragma unroll
+  for (int i = 0; i < 32; i += NV) unpack16<T>(*reinterpret_cast<const uint4*>(src + i), v + i);
+}
+
+// EPI: 0 Store, 1 StoreBias, 2 Accum, 3 SwigluFwd, 4 SwigluBwd (values of moe::Epi).
+template <int BN, bool A_MN, bool B_MN, int GROUP, int EPI, typename TC>
+__global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_constant__ Params p) {
+  using C = Cfg<BN>;
+  constexpr uint32_t kIdesc = make_idesc(BN, A_MN, B_MN);
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::kStages * C::kStageBytes);
+  uint64_t* full = bars;                       // [kStages]
+  uint64_t* empty = bars + C::kStages;         // [kStages]
+  uint64_t* tfull = bars + 2 * C::kStages;     // [2]
+  uint64_t* tempty = tfull + 2;                // [2]
+  uint64_t* done = tempty + 2;                 // [1]
+  uint32_t* s_tmem = reinterpret_cast<uint32_t*>(done + 1);
+  __shared__ int s_off[kMaxE + 1];
+  __shared__ int s_pref[kMaxE + 1];
+  __shared__ int s_total;
+  __shared__ volatile int s_abort;
+
+  const int tid = threadIdx.x;
+  const int warp = tid >> 5, lane = tid & 31;
+
+  if (warp == 0 && lane == 0) {
+    for (int s = 0; s < C::kStages; ++s) {
+      mbar_init(smem_u32(&full[s]), 1);
+      mbar_init(smem_u32(&empty[s]), 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(smem_u32(&tfull[a]), 1);
+      mbar_init(smem_u32(&tempty[a]), 4);
+    }
+    mbar_init(smem_u32(done), 1);
+    fence_barrier_init();
+    s_abort = 0;
+    tma_prefetch_desc(&p.ta);
+    tma_prefetch_desc(&p.tb);
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(s_tmem), C::kCols);
+    tmem_relinquish();
+  }
+  if (GROUP != 0) {
+    for (int i = tid; i <= p.num_groups; i += kThreads) s_off[i] = p.offsets[i];
+  }
+  __syncthreads();
+  if (tid == 0) {
+    if (GROUP == 0) {
+      s_total = p.tiles_m * p.tiles_n;
+    } else if (GROUP == 1) {
+      int acc = 0;
+      for (int g = 0; g < p.num_groups; ++g) {
+        s_pref[g] = acc;
+        acc += (s_off[g + 1] - s_off[g] + BM - 1) / BM;
+      }
+      s_pref[p.num_groups] = acc;
+      s_total = acc * p.tiles_n;
+    } else {
+      s_total = p.num_groups * p.tiles_m * p.tiles_n;
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *s_tmem;
+  const int total = s_total;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      int issued = 0;
+      uint32_t last_phase = 0;  // bit s: phase of the last copy issued into stage s
+      bool ok = true;
+      for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
+        Tile ti;
+        decode_tile<GROUP>(p, t, s_off, s_pref, ti);
+        const int64_t n0 = ti.n0 * BN;
+        for (int kb = 0; kb < ti.nkb; ++kb) {
+          if (!wait_bounded(smem_u32(&empty[stage]), phase ^ 1u, &s_abort, p.err)) { ok = false; break; }
+          const uint32_t fb = smem_u32(&full[stage]);
+          mbar_expect_tx(fb, C::kStageBytes);
+          const uint32_t sa = smem_u32(smem + stage * C::kStageBytes);
+          const uint32_t sb = sa + C::kABytes;
+          const int k0 = (int)(ti.kbeg + (int64_t)kb * BK);
+          if (A_MN) {
+            tma_load_2d(sa, &p.ta, fb, (int)ti.row0, k0);
+            tma_load_2d(sa + 8192, &p.ta, fb, (int)ti.row0 + 64, k0);
+          } else {
+            tma_load_2d(sa, &p.ta, fb, k0, (int)ti.row0);
+          }
+          if (B_MN) {
+            const int ky = (int)(ti.g * p.b_group_rows) + k0;
+#pragma unroll
+            for (int j = 0; j < BN / 64; ++j) tma_load_2d(sb + j * 8192, &p.tb, fb, (int)n0 + 64 * j, ky);
+          } else {
+            tma_load_2d(sb, &p.tb, fb, k0, (int)(ti.g * p.b_group_rows + n0));
+          }
+          last_phase = (last_phase & ~(1u << stage)) | (phase << stage);
+          ++issued;
+          if (++stage == C::kStages) { stage = 0; phase ^= 1u; }
+        }
+      }
+      // drain: every issued copy must land before the CTA exits
+      const int pending = issued < C::kStages ? issued : C::kStages;
+      for (int i = 0; i < pending; ++i) {
+        stage = (stage + C::kStages - 1) % C::kStages;
+        wait_drain(smem_u32(&full[stage]), (last_phase >> stage) & 1u, 1000000000ull);
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer
+    int stage = 0;
+    uint32_t phase = 0;
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    bool ok = true;
+    bool issued_any = false;
+    for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
+      Tile ti;
+      decode_tile<GROUP>(p, t, s_off, s_pref, ti);
+      if (ti.nkb == 0) continue;
+      issued_any = true;
+      if (!wait_bounded(smem_u32(&tempty[acc]), acc_phase ^ 1u, &s_abort, p.err)) { ok = false; break; }
+      tc_fence_after();
+      const uint32_t d_tmem = tmem_base + (uint32_t)(acc * BN);
+      for (int kb = 0; kb < ti.nkb; ++kb) {
+        if (!wait_bounded(smem_u32(&full[stage]), phase, &s_abort, p.err)) { ok = false; break; }
+        tc_fence_after();
+        uint8_t* sa_ptr = smem + stage * C::kStageBytes;
+        const uint32_t sa = smem_u32(sa_ptr);
+        const uint32_t sb = sa + C::kABytes;
+        if (GROUP == 2) {
+          // rows k >= kend of the last k-block belong to the next expert: zero them in A
+          const int64_t k0 = ti.kbeg + (int64_t)kb * BK;
+          const int valid = (int)imin64(BK, ti.kend - k0);
+          if (valid < BK) {
+            uint4 z = make_uint4(0, 0, 0, 0);
+            const int nrow = BK - valid;  // per chunk; 8 x 16 B per 128-byte row
+            for (int i = lane; i < 2 * nrow * 8; i += 32) {
+              const int chunk = i / (nrow * 8);
+              const int r = valid + (i % (nrow * 8)) / 8;
+              const int q = i % 8;
+              *reinterpret_cast<uint4*>(sa_ptr + chunk * 8192 + r * 128 + q * 16) = z;
+            }
+            fence_proxy_async_smem();
+          }
+          __syncwarp();
+        }
+        if (lane == 0) {
+#pragma unroll
+          for (int k = 0; k < BK / 16; ++k) {
+            uint64_t ad, bd;
+            if (A_MN) ad = make_sdesc(sa + k * 2048, 8192, 1024);
+            else ad = make_sdesc(sa + k * 32, 16, 1024);
+            if (B_MN) bd = make_sdesc(sb + k * 2048, 8192, 1024);
+            else bd = make_sdesc(sb + k * 32, 16, 1024);
+            mma_bf16(d_tmem, ad, bd, kIdesc, (kb > 0 || k > 0) ? 1u : 0u);
+          }
+          mma_commit(smem_u32(&empty[stage]));
+        }
+        __syncwarp();
+        if (++stage == C::kStages) { stage = 0; phase ^= 1u; }
+      }
+      if (!ok) break;
+      if (lane == 0) mma_commit(smem_u32(&tfull[acc]));
+      __syncwarp();
+      if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
+    }
+    // drain: all MMAs issued by this warp have completed before TMEM is freed
+    if (lane == 0 && issued_any) {
+      mma_commit(smem_u32(done));
+      wait_drain(smem_u32(done), 0, 1000000000ull);
+    }
+    __syncwarp();
+  } else {
+    // ------------------------------------------------------------ epilogue
+    const int q = warp & 3;
+    const int row_in_tile = q * 32 + lane;
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    for (int t = blockIdx.x; t < total; t += gridDim.x) {
+      Tile ti;
+      decode_tile<GROUP>(p, t, s_off, s_pref, ti);
+      const int64_t n0 = ti.n0 * BN;
+      const int64_t grow = ti.row0 + row_in_tile;
+      const bool vrow = grow < ti.row_end;
+      TC* Cb = static_cast<TC*>(p.C) + (GROUP == 2 ? (int64_t)ti.g * p.sc_g : 0);
+      if (ti.nkb == 0) {
+        // an expert with no rows: its weight-gradient tile is zero
+        if (vrow) {
+          float z[32];
+#pragma unroll
+          for (int i = 0; i < 32; ++i) z[i] = 0.f;
+          for (int c = 0; c < BN / 32; ++c) {
+            const int64_t col0 = n0 + c * 32;
+            if (col0 >= p.N) break;
+            store_row32<TC>(Cb + grow * p.ldc + col0, z, (int)imin64(32, p.N - col0));
+          }
+        }
+        continue;
+      }
+      if (!wait_bounded(smem_u32(&tfull[acc]), acc_phase, &s_abort, p.err)) break;
+      tc_fence_after();
+      const uint32_t tbase = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
+      float v[32];
+      if (EPI == 3) {
+        // packed [gate 64 | up 64] blocks: a = silu(g) * u
+        for (int blk = 0; blk < BN / 128; ++blk) {
+          const int64_t cb = n0 + blk * 128;
+          if (cb >= p.N) break;
+#pragma unroll 1
+          for (int half = 0; half < 2; ++half) {
+            float u[32];
+            tmem_ld32(tbase + blk * 128 + half * 32, v);
+            tmem_ld32(tbase + blk * 128 + 64 + half * 32, u);
+            if (vrow) {
+              TC* hrow = Cb + grow * p.ldc;
+              store_row32<TC>(hrow + cb + half * 32, v, 32);
+              store_row32<TC>(hrow + cb + 64 + half * 32, u, 32);
+              float a[32];
+#pragma unroll
+              for (int i = 0; i < 32; ++i) a[i] = silu_f(v[i]) * u[i];
+              TC* arow = static_cast<TC*>(p.aux) + grow * (p.N / 2);
+              store_row32<TC>(arow + cb / 2 + half * 32, a, 32);
+            }
+          }
+        }
+      } else {
+#pragma unroll 1
+        for (int c = 0; c < BN / 32; ++c) {
+          const int64_t col0 = n0 + c * 32;
+          if (col0 >= p.N) break;
+          tmem_ld32(tbase + c * 32, v);
+          if (!vrow) continue;
+          const int nvalid = (int)imin64(32, p.N - col0);
+          TC* crow = Cb + grow * p.ldc;
+          if (EPI == 0) {
+            store_row32<TC>(crow + col0, v, nvalid);
+          } else if (EPI == 1) {
+            if (p.bias) {
+#pragma unroll
+              for (int i = 0; i < 32; ++i)
+                if (i < nvalid) v[i] += p.bias[col0 + i];
+            }
+            store_row32<TC>(crow + col0, v, nvalid);
+          } else if (EPI == 2) {
+            if (nvalid == 32) {
+              float o[32];
+              load_row32<TC>(crow + col0, o);
+#pragma unroll
+              for (int i = 0; i < 32; ++i) v[i] += o[i];
+            } else {
+#pragma unroll
+              for (int i = 0; i < 32; ++i)
+                if (i < nvalid) v[i] += to_f32<TC>(crow[col0 + i]);
+            }
+            store_row32<TC>(crow + col0, v, nvalid);
+          } else if (EPI == 4) {
+            // v = dA for features col0 .. col0 + 31; gate / up columns in the packed order
+            const int64_t cg = (col0 / 64) * 128 + (col0 % 64);
+            const TC* hrow = static_cast<const TC*>(p.h_in) + grow * p.ldc;
+            float g[32], u[32], dg[32], du[32];
+            load_row32<TC>(hrow + cg, g);
+            load_row32<TC>(hrow + cg + 64, u);
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+              const float sg = sigmoid_f(g[i]);
+              dg[i] = v[i] * u[i] * sg * (1.0f + g[i] * (1.0f - sg));
+              du[i] = v[i] * g[i] * sg;
+            }
+            store_row32<TC>(crow + cg, dg, 32);
+            store_row32<TC>(crow + cg + 64, du, 32);
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_u32(&tempty[acc]));
+      if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc(tmem_base, C::kCols);
+}
+
+}  // namespace tc
+}  // namespace moe
