@@ -65,7 +65,8 @@ typedef enum {
     MOE_ERR_WORKSPACE = -5,   /* ws_bytes smaller than moe_workspace_size() */
     MOE_ERR_CUDA = -6,        /* a CUDA runtime call or launch failed (see moe_last_cuda_error) */
     MOE_ERR_DEVICE = -7,      /* the device status word is set (moe_check_device_status) */
-    MOE_ERR_UNSUPPORTED = -8  /* valid request this build does not implement */
+    MOE_ERR_UNSUPPORTED = -8, /* valid request this build does not implement */
+    MOE_ERR_TOO_LARGE = -9    /* shape exceeds the fixed scratch of moe_dispatch_noalloc */
 } moe_status;
 
 typedef enum { MOE_BF16 = 0, MOE_F32 = 1 } moe_dtype;
@@ -112,6 +113,34 @@ int moe_topk(const moe_shape_t* shape, const float* logits, int32_t* topk_idx, f
 int moe_dispatch(const moe_shape_t* shape, const void* x, const int32_t* topk_idx, const float* topk_prob,
                  int32_t* expert_offsets, int32_t* row_of_slot, int32_t* token_of_row,
                  void* x_perm, float* prob_perm, void* ws, size_t ws_bytes, void* stream);
+
+/* Dispatch that allocates nothing and takes no workspace.  The paper has no
+ * counterpart: this entry point exists for callers that cannot allocate
+ * device memory when they call the layer -- a host framework that has already
+ * reserved all device memory for its own pool or forbids allocation inside its
+ * step loop, or a runtime that cannot afford cudaMalloc's implicit device-wide
+ * synchronisation -- and so cannot provide the workspace moe_dispatch needs.
+ *
+ * Results are identical to moe_dispatch (same arguments minus ws/ws_bytes).
+ * The counting sort's per-chunk histogram and prefix-sum tables,
+ * 2 * E * ceil(T*K / 2048) int32 values, live in one fixed device array of
+ * MOE_DISPATCH_NOALLOC_SCRATCH_INTS int32 (1 MiB) compiled into the library;
+ * every GPU that loads the library holds its copy until the process exits.
+ * The call makes no cudaMalloc / cudaFree or other allocating call.
+ *  - A shape whose tables do not fit (E * ceil(T*K / 2048) > 131072) returns
+ *    MOE_ERR_TOO_LARGE before anything is enqueued.
+ *  - The first call on a device looks up that device's copy of the array
+ *    (cudaGetSymbolAddress, with the device current); make that first call
+ *    before any stream capture on the device.
+ *  - All calls share the one array.  Each call writes every table entry it
+ *    reads before reading it, so nothing from an earlier call leaks into a
+ *    result; but calls whose kernels overlap on the GPU (different streams or
+ *    host threads without ordering between them) race on the array, and the
+ *    caller must order them. */
+#define MOE_DISPATCH_NOALLOC_SCRATCH_INTS 262144
+int moe_dispatch_noalloc(const moe_shape_t* shape, const void* x, const int32_t* topk_idx,
+                         const float* topk_prob, int32_t* expert_offsets, int32_t* row_of_slot,
+                         int32_t* token_of_row, void* x_perm, float* prob_perm, void* stream);
 
 /* Grouped SwiGLU expert FFN (Sec. 5.2 grouped GEMM; reading R6): for every
  * expert e and its rows, h = x_perm . w1_e^T ([rows, 2F], packed order),

@@ -22,6 +22,7 @@ MOE_F32 = 1
 STATUS = {
     0: "MOE_OK", -1: "MOE_ERR_SHAPE", -2: "MOE_ERR_DTYPE", -3: "MOE_ERR_ALIGN", -4: "MOE_ERR_NULL",
     -5: "MOE_ERR_WORKSPACE", -6: "MOE_ERR_CUDA", -7: "MOE_ERR_DEVICE", -8: "MOE_ERR_UNSUPPORTED",
+    -9: "MOE_ERR_TOO_LARGE",
 }
 
 # Every symbol include/moe.h declares.
@@ -30,7 +31,7 @@ EXPORTS = (
     "moe_combine_bwd", "moe_expert_ffn_bwd", "moe_dispatch_bwd", "moe_route_bwd", "moe_latent_proj",
     "moe_latent_proj_bwd", "moe_pack_w1", "moe_eq1_bytes", "moe_check_device_status",
     "moe_device_status_word", "moe_last_cuda_error", "moe_strerror", "moe_version", "moe_prof_enable",
-    "moe_prof_reset", "moe_prof_count", "moe_prof_get", "moe_launch_count",
+    "moe_prof_reset", "moe_prof_count", "moe_prof_get", "moe_launch_count", "moe_dispatch_noalloc",
 )
 
 
@@ -95,6 +96,7 @@ _SIGS = {
     "moe_prof_get": ([ctypes.c_int, ctypes.POINTER(ctypes.c_char_p), ctypes.POINTER(ctypes.c_int),
                       ctypes.POINTER(ctypes.c_double)], ctypes.c_int),
     "moe_launch_count": ([], ctypes.c_uint64),
+    "moe_dispatch_noalloc": ([_SHP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP], ctypes.c_int),
 }
 
 
@@ -176,6 +178,15 @@ def moe_dispatch(shape, x, topk_idx, topk_prob, expert_offsets, row_of_slot, tok
     _check("moe_dispatch", lib().moe_dispatch(_shape(shape), _p(x), _p(topk_idx), _p(topk_prob), _p(expert_offsets),
                                               _p(row_of_slot), _p(token_of_row), _p(x_perm), _p(prob_perm), _p(ws),
                                               _nbytes(ws), _stream(stream)))
+
+
+def moe_dispatch_noalloc(shape, x, topk_idx, topk_prob, expert_offsets, row_of_slot, token_of_row, x_perm,
+                         prob_perm, stream=None):
+    """moe_dispatch without a workspace, for callers that cannot allocate device
+    memory at the call (the scratch is a fixed 1 MiB array inside the library)."""
+    _check("moe_dispatch_noalloc", lib().moe_dispatch_noalloc(
+        _shape(shape), _p(x), _p(topk_idx), _p(topk_prob), _p(expert_offsets), _p(row_of_slot), _p(token_of_row),
+        _p(x_perm), _p(prob_perm), _stream(stream)))
 
 
 def moe_expert_ffn(shape, x_perm, expert_offsets, w1, w2, h_save, act_save, y_perm, ws, stream=None):

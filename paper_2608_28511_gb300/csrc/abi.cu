@@ -217,6 +217,27 @@ void prof_end(const char* name, cudaStream_t s) {
 
 void count_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
 
+int abi_check_shape(const moe_shape_t* s, ShapeInfo* out) {
+  Dims d;
+  const int st = check_shape(s, &d);
+  if (st != MOE_OK) return st;
+  out->T = d.T;
+  out->TK = d.TK;
+  out->K = d.K;
+  out->D = d.D;
+  out->E = d.E;
+  out->F = d.F;
+  out->H = d.H;
+  out->Din = d.Din;
+  out->dt = d.dt;
+  out->bx = d.bx;
+  return MOE_OK;
+}
+
+int abi_device_ctx(void* stream, Ctx* c) { return get_ctx(stream, c); }
+
+int abi_cuda_status(cudaError_t e) { return cuda_status(e); }
+
 }  // namespace moe
 
 using namespace moe;
@@ -236,6 +257,7 @@ const char* moe_strerror(int status) {
     case MOE_ERR_CUDA: return "CUDA runtime error (see moe_last_cuda_error)";
     case MOE_ERR_DEVICE: return "device status word set (out-of-range expert index or expired bounded wait)";
     case MOE_ERR_UNSUPPORTED: return "unsupported request";
+    case MOE_ERR_TOO_LARGE: return "shape exceeds the fixed scratch of moe_dispatch_noalloc (E * ceil(T*K/2048) > 131072)";
     default: return "unknown status";
   }
 }

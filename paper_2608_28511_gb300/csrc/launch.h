@@ -5,6 +5,8 @@
 #include <stdint.h>
 #include <stddef.h>
 
+#include "moe.h"
+
 namespace moe {
 
 struct Ctx {
@@ -29,6 +31,18 @@ struct KernelScope {
 enum class DType : int { BF16 = 0, F32 = 1 };
 
 inline size_t dsize(DType t) { return t == DType::BF16 ? 2 : 4; }
+
+// Shape validation and per-device context shared by the entry points
+// (implemented in abi.cu).
+struct ShapeInfo {
+  int64_t T, TK;
+  int K, D, E, F, H, Din;
+  DType dt;
+  size_t bx;
+};
+int abi_check_shape(const moe_shape_t* s, ShapeInfo* d);
+int abi_device_ctx(void* stream, Ctx* c);
+int abi_cuda_status(cudaError_t e);
 
 // ---------------------------------------------------------------------------
 // router.cu
