@@ -133,34 +133,72 @@ class ClockSampler:
 # Oracle timing on the host cores (cpu_baseline and the reference arm)
 # ---------------------------------------------------------------------------
 
-def oracle_step(w: synth.Workload, T_sample: int, seed: int = 0) -> float:
-    """One oracle forward + backward over T_sample tokens of workload w; returns seconds."""
-    import oracle as O
-    inp = synth.make_inputs(w, seed=seed, T=T_sample)
-    o = {k: synth.to_f64(v) for k, v in inp.items()}
-    t0 = time.perf_counter()
-    fwd = O.layer_forward(o["x"], o["w_router"], o["w_gate"], o["w_up"], o["w2"], w.K, bias=o["bias"],
-                          w_down=o.get("w_down"), w_upp=o.get("w_upp"))
-    O.layer_backward(fwd, o["dy"], o["x"], o["w_router"], o["w_gate"], o["w_up"], o["w2"],
-                     w_down=o.get("w_down"), w_upp=o.get("w_upp"))
-    return time.perf_counter() - t0
+class OracleRunner:
+    """The float64 oracle on the host cores over a bounded token sample of a
+    workload: inputs are drawn and widened to float64 once; each step times one
+    oracle forward + backward over ``T_sample`` fresh tokens (weights shared)."""
+
+    def __init__(self, w: synth.Workload, T_pool: int, seed: int = 0):
+        import oracle as O
+        self.O = O
+        self.w = w
+        inp = synth.make_inputs(w, seed=seed, T=T_pool)
+        self.o = {k: synth.to_f64(v) for k, v in inp.items()}
+        self.T_pool = T_pool
+        self.cursor = 0
+
+    def step(self, T_sample: int) -> float:
+        o, w, O = self.o, self.w, self.O
+        if self.cursor + T_sample > self.T_pool:
+            self.cursor = 0
+        sl = slice(self.cursor, self.cursor + T_sample)
+        self.cursor += T_sample
+        x, dy = o["x"][sl], o["dy"][sl]
+        t0 = time.perf_counter()
+        fwd = O.layer_forward(x, o["w_router"], o["w_gate"], o["w_up"], o["w2"], w.K, bias=o["bias"],
+                              w_down=o.get("w_down"), w_upp=o.get("w_upp"))
+        O.layer_backward(fwd, dy, x, o["w_router"], o["w_gate"], o["w_up"], o["w2"],
+                         w_down=o.get("w_down"), w_upp=o.get("w_upp"))
+        return time.perf_counter() - t0
 
 
-def cpu_baseline(w: synth.Workload, T_sample: int, repeats: int = 2) -> dict:
-    ts = [oracle_step(w, T_sample, seed=i) for i in range(repeats)]
+def _threads() -> int:
+    for var in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS"):
+        v = os.environ.get(var)
+        if v and v.isdigit():
+            return int(v)
+    return os.cpu_count() or 1
+
+
+def cpu_baseline(w: synth.Workload, budget_s: float = 15.0) -> dict:
+    """Oracle throughput on a bounded sample (about ``budget_s`` of CPU work)."""
+    runner = OracleRunner(w, T_pool=2048, seed=99)
+    probe = 32
+    t_probe = runner.step(probe)
+    T_sample = int(max(32, min(2048, probe * budget_s / 2 / max(t_probe, 1e-3))))
+    ts = [runner.step(T_sample) for _ in range(2)]
     sec = statistics.median(ts)
-    return {"value": T_sample / sec, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
-            "sample": f"{w.name} shapes with {T_sample} tokens, float64 NumPy oracle fwd+bwd, median of {repeats}"}
+    return {"value": T_sample / sec, "unit": UNIT, "cores": _threads(), "kind": "oracle",
+            "sample": f"{w.name} shapes and weights, {T_sample} tokens, float64 NumPy oracle forward+backward, "
+                      f"median of 2 runs"}
 
 
 def run_reference(args, w: synth.Workload) -> None:
+    """The oracle as it stands on the host cores: each step a token sample of
+    the workload sized so that warm-up + steps take about two minutes."""
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return
-    T_sample = args.ref_tokens
+    runner = OracleRunner(w, T_pool=2048, seed=1)
+    probe = 16
+    t_probe = runner.step(probe)
+    per_step = 120.0 / max(1, args.steps + args.warmup)
+    T_sample = int(max(4, min(1024, probe * per_step / max(t_probe, 1e-3))))
+    if args.ref_tokens:
+        T_sample = args.ref_tokens
     for _ in range(args.warmup):
-        oracle_step(w, T_sample)
-    ts = [oracle_step(w, T_sample, seed=i + 1) for i in range(args.steps)]
+        runner.step(T_sample)
+    ts = [runner.step(T_sample) for _ in range(args.steps)]
     tot = sum(ts)
     value = T_sample * args.steps / tot
     line = {
@@ -168,8 +206,8 @@ def run_reference(args, w: synth.Workload) -> None:
         "warmup": args.warmup, "ms_per_step": 1e3 * tot / args.steps, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "config": {"workload": w.name, "T_sample": T_sample, "note": "float64 CPU oracle on host cores"},
-        "cpu_baseline": {"value": value, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
-                         "sample": f"{w.name} shapes, {T_sample} tokens per step"},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": _threads(), "kind": "oracle",
+                         "sample": f"{w.name} shapes and weights, {T_sample} tokens per step"},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
@@ -182,12 +220,12 @@ def run_reference(args, w: synth.Workload) -> None:
 def main() -> None:
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=300)
+    ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--workload", default="C2")
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
-    ap.add_argument("--ref-tokens", type=int, default=64)
-    ap.add_argument("--cpu-tokens", type=int, default=256)
+    ap.add_argument("--ref-tokens", type=int, default=0, help="fixed oracle tokens per step (0 = sized to time)")
+    ap.add_argument("--cpu-budget", type=float, default=15.0, help="seconds of CPU work for cpu_baseline")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=10)
     args = ap.parse_args()
@@ -260,28 +298,32 @@ def main() -> None:
     assert abi.moe_check_device_status() == 0
 
     # ---- end to end through the public API with host buffers
-    x_h = inputs["x"].pin_memory()
-    dy_h = inputs["dy"].pin_memory()
-    y_h = torch.empty_like(x_h).pin_memory()
-    dx_h = torch.empty_like(x_h).pin_memory()
-    h2d = x_h.numel() * x_h.element_size() + dy_h.numel() * dy_h.element_size()
-    d2h = y_h.numel() * y_h.element_size() + dx_h.numel() * dx_h.element_size()
-    e_s, e_e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    for i in range(args.e2e_steps + 2):
-        if i == 2:
-            e_s.record(stream)
-        L.x.copy_(x_h, non_blocking=True)
-        L.dy.copy_(dy_h, non_blocking=True)
-        L.step()
-        y_h.copy_(L.y, non_blocking=True)
-        dx_h.copy_(L.dx, non_blocking=True)
-    e_e.record(stream)
-    torch.cuda.synchronize()
-    e2e_ms = e_s.elapsed_time(e_e) / args.e2e_steps
-    if world > 1:
-        tt = torch.tensor([e2e_ms], device="cuda", dtype=torch.float64)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        e2e_ms = float(tt.item())
+    e2e = None
+    if args.e2e_steps > 0:
+        x_h = inputs["x"].pin_memory()
+        dy_h = inputs["dy"].pin_memory()
+        y_h = torch.empty_like(x_h).pin_memory()
+        dx_h = torch.empty_like(x_h).pin_memory()
+        h2d = x_h.numel() * x_h.element_size() + dy_h.numel() * dy_h.element_size()
+        d2h = y_h.numel() * y_h.element_size() + dx_h.numel() * dx_h.element_size()
+        e_s, e_e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        for i in range(args.e2e_steps + 2):
+            if i == 2:
+                e_s.record(stream)
+            L.x.copy_(x_h, non_blocking=True)
+            L.dy.copy_(dy_h, non_blocking=True)
+            L.step()
+            y_h.copy_(L.y, non_blocking=True)
+            dx_h.copy_(L.dx, non_blocking=True)
+        e_e.record(stream)
+        torch.cuda.synchronize()
+        e2e_ms = e_s.elapsed_time(e_e) / args.e2e_steps
+        if world > 1:
+            tt = torch.tensor([e2e_ms], device="cuda", dtype=torch.float64)
+            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+            e2e_ms = float(tt.item())
+        e2e = {"value": world * T / (e2e_ms * 1e-3), "unit": UNIT, "h2d_bytes_per_step": h2d,
+               "d2h_bytes_per_step": d2h}
 
     # ---- per-kernel roofline from the live events
     peaks = _peaks()
@@ -324,7 +366,7 @@ def main() -> None:
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        cpu = cpu_baseline(w, args.cpu_tokens)
+        cpu = cpu_baseline(w, args.cpu_budget)
 
     if rank == 0:
         line = {
@@ -339,8 +381,7 @@ def main() -> None:
             "dispatch_gbs": permute_family_bytes(w, T) / (perm_ms * 1e-3) / 1e9 if perm_ms else None,
             "expert_tflops": expert_flops(w, T) / (exp_ms * 1e-3) / 1e12 if exp_ms else None,
             "cpu_baseline": cpu,
-            "e2e": {"value": world * T / (e2e_ms * 1e-3), "unit": UNIT, "h2d_bytes_per_step": h2d,
-                    "d2h_bytes_per_step": d2h},
+            "e2e": e2e,
             "gpu_launches": launches * args.steps,
             "gpu_launches_per_step": launches,
             "clocks": clk,
