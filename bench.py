@@ -342,7 +342,10 @@ def main() -> None:
             tr = json.load(f)
         ent = tr.get(w.name, {}).get(tname)
         if ent is not None:
-            traffic = ent
+            import hashlib
+            src = os.path.join(ROOT, ent["src"])
+            sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16] if os.path.exists(src) else None
+            traffic = ent["bytes"] if sha == ent["sha256_16"] else None   # stale once the kernel changed
     if tk["bound"] == "tensor":
         achieved = tk["work_per_launch"] / (tk["avg_launch_ms"] * 1e-3) / 1e12
         peak = peaks["bf16_tflops_sustained"]

@@ -120,9 +120,10 @@ def test_full_size_parity(cfg):
         wg, wu, w2 = _w64(inp["w_gate"][e]), _w64(inp["w_up"][e]), _w64(inp["w2"][e])
         g, u, a, Y = O.expert_ffn_one(X_e, wg, wu, w2)
         _, dwg, dwu, dw2 = O.expert_ffn_bwd_one(pe * dY_e, X_e, g, u, wg, wu, w2)
-        gg, gu = L.unpack_w1_like(L.dw1[e:e + 1].contiguous())
-        assert rel_frob(f64(gg[0]), dwg) <= REL_FROB, e
-        assert rel_frob(f64(gu[0]), dwu) <= REL_FROB, e
+        v = L.dw1[e].view(w.F // 64, 2, 64, w.D)
+        gg, gu = v[:, 0].reshape(w.F, w.D), v[:, 1].reshape(w.F, w.D)
+        assert rel_frob(f64(gg), dwg) <= REL_FROB, e
+        assert rel_frob(f64(gu), dwu) <= REL_FROB, e
         assert rel_frob(f64(L.dw2[e]), dw2) <= REL_FROB, e
     for e in np.nonzero(cnt == 0)[0][:4]:
         assert float(L.dw1[e].abs().max()) == 0.0 and float(L.dw2[e].abs().max()) == 0.0
