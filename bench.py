@@ -214,6 +214,31 @@ def run_reference(args, w: synth.Workload) -> None:
 
 
 # ---------------------------------------------------------------------------
+# Multi-rank host logic (weak scaling: every rank its own tokens)
+# ---------------------------------------------------------------------------
+
+def rank_seed(w: synth.Workload, rank: int) -> int:
+    """Seed of rank ``rank``'s token batch: ranks hold disjoint synthetic batches."""
+    return w.seed + rank
+
+
+def max_over_ranks(value: float, world: int, device: str) -> float:
+    """The slowest rank's time sets the job's time (a timing collective only)."""
+    if world <= 1:
+        return value
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([value], device=device, dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(world: int, T: int, t_max_ms: float) -> float:
+    """Whole-job routed tokens per second: all ranks' tokens over the slowest rank's time."""
+    return world * T / (t_max_ms * 1e-3)
+
+
+# ---------------------------------------------------------------------------
 # GPU arm
 # ---------------------------------------------------------------------------
 
@@ -252,7 +277,7 @@ def main() -> None:
     from paper_2608_28511_gb300.layer import MoeLayer
 
     T = w.T
-    inputs = synth.make_inputs(w, seed=w.seed + rank)      # each rank its own tokens
+    inputs = synth.make_inputs(w, seed=rank_seed(w, rank))      # each rank its own tokens
     L = MoeLayer(w.S, w.GBS, w.K, w.D, w.E, w.F, w.dtype, w.H)
     L.load(inputs)
     stream = torch.cuda.current_stream()
@@ -290,11 +315,7 @@ def main() -> None:
     abi.moe_prof_enable(False)
     prof = abi.moe_prof_read()
     step_ms = sum(s.elapsed_time(e) for s, e in zip(ev_s, ev_e)) / args.steps
-    t_max = step_ms
-    if world > 1:
-        tt = torch.tensor([step_ms], device="cuda", dtype=torch.float64)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        t_max = float(tt.item())
+    t_max = max_over_ranks(step_ms, world, "cuda")
     assert abi.moe_check_device_status() == 0
 
     # ---- end to end through the public API with host buffers
@@ -317,12 +338,8 @@ def main() -> None:
             dx_h.copy_(L.dx, non_blocking=True)
         e_e.record(stream)
         torch.cuda.synchronize()
-        e2e_ms = e_s.elapsed_time(e_e) / args.e2e_steps
-        if world > 1:
-            tt = torch.tensor([e2e_ms], device="cuda", dtype=torch.float64)
-            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-            e2e_ms = float(tt.item())
-        e2e = {"value": world * T / (e2e_ms * 1e-3), "unit": UNIT, "h2d_bytes_per_step": h2d,
+        e2e_ms = max_over_ranks(e_s.elapsed_time(e_e) / args.e2e_steps, world, "cuda")
+        e2e = {"value": job_throughput(world, T, e2e_ms), "unit": UNIT, "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": d2h}
 
     # ---- per-kernel roofline from the live events
@@ -373,7 +390,7 @@ def main() -> None:
 
     if rank == 0:
         line = {
-            "metric": METRIC, "value": world * T / (t_max * 1e-3), "unit": UNIT, "n_gpus": world,
+            "metric": METRIC, "value": job_throughput(world, T, t_max), "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": t_max, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
             "config": {"workload": w.name, "T": T, "S": w.S, "GBS": w.GBS, "D": w.D, "E": w.E, "K": w.K, "F": w.F,

@@ -1,0 +1,70 @@
+"""Multi-rank host logic of bench.py on CPU with the gloo backend (world size 2).
+
+The layer shards by tokens with no data-path exchange: each rank draws its own
+batch (seed + rank), the job time is the slowest rank's (a max-reduce, the only
+collective besides the barrier), and throughput counts every rank's tokens.
+"""
+import os
+import socket
+
+import pytest
+import torch
+import torch.distributed as dist
+import torch.multiprocessing as mp
+
+import bench
+import synth
+
+
+def _free_port() -> int:
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+def _worker(rank, world, port, q):
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), RANK=str(rank), WORLD_SIZE=str(world))
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        w = synth.Workload("mr", S=16, GBS=2, D=64, E=4, K=2, F=64)
+        x = synth.make_inputs(w, seed=bench.rank_seed(w, rank))["x"]
+        xs = [torch.empty_like(x) for _ in range(world)]
+        dist.all_gather(xs, x)                        # test-only: compare the ranks' batches
+        distinct = not torch.equal(xs[0], xs[1])
+        t = bench.max_over_ranks(1.0 + rank, world, "cpu")
+        dist.barrier()
+        q.put((rank, distinct, t, bench.job_throughput(world, w.T, t)))
+    finally:
+        dist.destroy_process_group()
+
+
+def test_two_gloo_ranks_shard_tokens_and_take_the_slowest_time():
+    world = 2
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_worker, args=(r, world, port, q)) for r in range(world)]
+    for p in procs:
+        p.start()
+    for p in procs:
+        p.join(timeout=120)
+        assert p.exitcode == 0
+    res = sorted(q.get(timeout=10) for _ in range(world))
+    for rank, distinct, t, thr in res:
+        assert distinct                              # each rank holds its own tokens
+        assert t == 2.0                              # the slowest rank's time on every rank
+        assert thr == pytest.approx(world * 32 / 2e-3)
+
+
+def test_reference_arm_runs_only_on_rank_zero(monkeypatch, capsys):
+    monkeypatch.setenv("RANK", "1")
+    monkeypatch.setattr(bench, "OracleRunner", lambda *a, **k: pytest.fail("rank 1 must not run the oracle"))
+
+    class A:
+        steps, warmup, ref_tokens, gpus = 3, 3, 0, 2
+    bench.run_reference(A(), synth.TINY)
+    assert capsys.readouterr().out == ""
+
+
+def test_job_throughput_is_weak_scaling():
+    assert bench.job_throughput(4, 8192, 2.0) == pytest.approx(4 * bench.job_throughput(1, 8192, 2.0))
