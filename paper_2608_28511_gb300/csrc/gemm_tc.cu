@@ -75,7 +75,7 @@ bool make_plan(const GemmDesc& d, Plan* pl) {
   switch (d.epi) {
     case Epi::Store: break;
     case Epi::StoreBias: if (d.c_type != DType::F32) return false; break;
-    case Epi::Accum: if (d.c_type != DType::BF16) return false; break;
+    case Epi::Accum: if (d.c_type != DType::BF16 || d.N % 64) return false; break;
     case Epi::SwigluFwd:
       if (d.c_type != DType::BF16 || d.N % 128 || !d.aux || !al16(d.aux)) return false;
       break;

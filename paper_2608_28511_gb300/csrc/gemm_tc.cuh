@@ -199,8 +199,109 @@ struct Cfg {
   static constexpr int kStageBytes = kABytes + kBBytes;
   static constexpr int kStages = (196608 / kStageBytes) < 8 ? (196608 / kStageBytes) : 8;
   static constexpr int kCols = 2 * BN;  // double-buffered fp32 accumulator
-  static constexpr int kSmem = kStages * kStageBytes + 1024 /*align*/ + 512 /*barriers*/;
+  // per epilogue warp: 32 rows x 128 B staging, rows padded to 144 B (conflict-free both ways)
+  static constexpr int kPitch = 144;
+  static constexpr int kStageBufBytes = 32 * kPitch;
+  static constexpr int kStagingBytes = 4 * kStageBufBytes;
+  static constexpr int kSmem = kStages * kStageBytes + kStagingBytes + 1024 /*align*/ + 512 /*barriers*/;
 };
+
+// ---------------------------------------------------------------------------
+// Epilogue staging: each epilogue warp owns 32 accumulator rows (one per
+// lane).  A lane writes its row into the warp's staging buffer, then the warp
+// copies the 32 rows to global memory with lanes covering consecutive 16-byte
+// pieces of a row, so every store instruction writes whole 128-byte lines
+// instead of 32 scattered half-sectors.  Loads of epilogue inputs (the saved
+// h, an accumulation target) take the reverse path.
+// ---------------------------------------------------------------------------
+template <int NB>  // bytes per row: 64 or 128
+__device__ __forceinline__ void stage_put(uint8_t* buf, int lane, const uint4* row) {
+#pragma unroll
+  for (int j = 0; j < NB / 16; ++j) *reinterpret_cast<uint4*>(buf + lane * 144 + j * 16) = row[j];
+}
+template <int NB>
+__device__ __forceinline__ void stage_get(const uint8_t* buf, int lane, uint4* row) {
+#pragma unroll
+  for (int j = 0; j < NB / 16; ++j) row[j] = *reinterpret_cast<const uint4*>(buf + lane * 144 + j * 16);
+}
+// buf rows 0..31 -> gbase + r * ld_bytes (rows r >= nrows are skipped).
+template <int NB>
+__device__ __forceinline__ void stage_store(const uint8_t* buf, int lane, uint8_t* gbase, int64_t ld_bytes,
+                                            int nrows) {
+  constexpr int CPR = NB / 16, RPI = 32 / CPR;
+#pragma unroll
+  for (int it = 0; it < 32 / RPI; ++it) {
+    const int r = it * RPI + lane / CPR, c = lane % CPR;
+    const uint4 v = *reinterpret_cast<const uint4*>(buf + r * 144 + c * 16);
+    if (r < nrows) *reinterpret_cast<uint4*>(gbase + r * ld_bytes + c * 16) = v;
+  }
+}
+// Pieces of the 32-row block an EPI 2 / EPI 4 chunk reads, fetched into
+// registers (16 bytes per piece, rows >= nrows as zero).  EPI 2: 32 bf16
+// columns of C at col0 (4 pieces per lane).  EPI 4: the gate columns
+// cg .. cg+31 and up columns cg+64 .. cg+95 of h for features col0 .. col0+31
+// (8 pieces per lane; a staging row holds gate bytes 0..63, up bytes 64..127).
+template <int EPI>
+__device__ __forceinline__ void epi_fetch(const uint8_t* rows, int64_t ld_b, int64_t col0, int lane, int nrows,
+                                          uint4* dst) {
+  if (EPI == 4) {
+    const int64_t cg = (col0 / 64) * 128 + (col0 % 64);
+#pragma unroll
+    for (int it = 0; it < 8; ++it) {
+      const int r = it * 4 + lane / 8, pc = lane % 8;
+      const int64_t off = pc < 4 ? cg * 2 + pc * 16 : (cg + 64) * 2 + (pc - 4) * 16;
+      dst[it] = r < nrows ? *reinterpret_cast<const uint4*>(rows + r * ld_b + off) : make_uint4(0, 0, 0, 0);
+    }
+  } else {
+#pragma unroll
+    for (int it = 0; it < 4; ++it) {
+      const int r = it * 8 + lane / 4, pc = lane % 4;
+      dst[it] = r < nrows ? *reinterpret_cast<const uint4*>(rows + r * ld_b + col0 * 2 + pc * 16)
+                          : make_uint4(0, 0, 0, 0);
+    }
+  }
+}
+template <int EPI>
+__device__ __forceinline__ void epi_put(uint8_t* buf, int lane, const uint4* src) {
+  if (EPI == 4) {
+#pragma unroll
+    for (int it = 0; it < 8; ++it) {
+      const int r = it * 4 + lane / 8, pc = lane % 8;
+      *reinterpret_cast<uint4*>(buf + r * 144 + pc * 16) = src[it];
+    }
+  } else {
+#pragma unroll
+    for (int it = 0; it < 4; ++it) {
+      const int r = it * 8 + lane / 4, pc = lane % 4;
+      *reinterpret_cast<uint4*>(buf + r * 144 + pc * 16) = src[it];
+    }
+  }
+}
+// Staging rows [dg 64 B | du 64 B] -> dH gate and up columns of features col0 .. col0+31.
+__device__ __forceinline__ void epi_store_gu(const uint8_t* buf, int lane, uint8_t* rows, int64_t ld_b,
+                                             int64_t col0, int nrows) {
+  const int64_t cg = (col0 / 64) * 128 + (col0 % 64);
+#pragma unroll
+  for (int it = 0; it < 8; ++it) {
+    const int r = it * 4 + lane / 8, pc = lane % 8;
+    const int64_t off = pc < 4 ? cg * 2 + pc * 16 : (cg + 64) * 2 + (pc - 4) * 16;
+    const uint4 v = *reinterpret_cast<const uint4*>(buf + r * 144 + pc * 16);
+    if (r < nrows) *reinterpret_cast<uint4*>(rows + r * ld_b + off) = v;
+  }
+}
+// gbase + r * ld_bytes -> buf rows 0..31 (rows r >= nrows read as zero).
+template <int NB>
+__device__ __forceinline__ void stage_load(uint8_t* buf, int lane, const uint8_t* gbase, int64_t ld_bytes,
+                                           int nrows) {
+  constexpr int CPR = NB / 16, RPI = 32 / CPR;
+#pragma unroll
+  for (int it = 0; it < 32 / RPI; ++it) {
+    const int r = it * RPI + lane / CPR, c = lane % CPR;
+    uint4 v = make_uint4(0, 0, 0, 0);
+    if (r < nrows) v = *reinterpret_cast<const uint4*>(gbase + r * ld_bytes + c * 16);
+    *reinterpret_cast<uint4*>(buf + r * 144 + c * 16) = v;
+  }
+}
 
 struct Tile {
   int g;
@@ -248,6 +349,7 @@ __device__ __forceinline__ void decode_tile(const Params& p, int t, const int* s
 }
 
 __device__ __forceinline__ int64_t imin64(int64_t a, int64_t b) { return a < b ? a : b; }
+__device__ __forceinline__ int64_t imax64(int64_t a, int64_t b) { return a > b ? a : b; }
 
 __device__ __forceinline__ float silu_f(float v) { return v / (1.0f + __expf(-v)); }
 __device__ __forceinline__ float sigmoid_f(float v) { return 1.0f / (1.0f + __expf(-v)); }
@@ -278,7 +380,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
   constexpr uint32_t kIdesc = make_idesc(BN, A_MN, B_MN);
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::kStages * C::kStageBytes);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::kStages * C::kStageBytes + C::kStagingBytes);
   uint64_t* full = bars;                       // [kStages]
   uint64_t* empty = bars + C::kStages;         // [kStages]
   uint64_t* tfull = bars + 2 * C::kStages;     // [2]
@@ -449,55 +551,141 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
   } else {
     // ------------------------------------------------------------ epilogue
     const int q = warp & 3;
-    const int row_in_tile = q * 32 + lane;
+    uint8_t* stg = smem + C::kStages * C::kStageBytes + q * C::kStageBufBytes;
+    constexpr int RB = (int)sizeof(TC) * 32;  // bytes of 32 columns of C
+    constexpr int NP = RB / 16;               // 16-byte pieces per 32 columns
+    const int64_t ldc_b = p.ldc * (int64_t)sizeof(TC);
     int acc = 0;
     uint32_t acc_phase = 0;
     for (int t = blockIdx.x; t < total; t += gridDim.x) {
       Tile ti;
       decode_tile<GROUP>(p, t, s_off, s_pref, ti);
       const int64_t n0 = ti.n0 * BN;
-      const int64_t grow = ti.row0 + row_in_tile;
-      const bool vrow = grow < ti.row_end;
+      const int64_t rbase = ti.row0 + q * 32;  // this warp's first row
+      const int nrows = (int)imax64(0, imin64(32, ti.row_end - rbase));
+      const int64_t grow = rbase + lane;
+      const bool vrow = lane < nrows;
       TC* Cb = static_cast<TC*>(p.C) + (GROUP == 2 ? (int64_t)ti.g * p.sc_g : 0);
+      uint8_t* c_rows = reinterpret_cast<uint8_t*>(Cb) + rbase * ldc_b;
       if (ti.nkb == 0) {
         // an expert with no rows: its weight-gradient tile is zero
-        if (vrow) {
-          float z[32];
+        uint4 z[NP];
 #pragma unroll
-          for (int i = 0; i < 32; ++i) z[i] = 0.f;
-          for (int c = 0; c < BN / 32; ++c) {
-            const int64_t col0 = n0 + c * 32;
-            if (col0 >= p.N) break;
-            store_row32<TC>(Cb + grow * p.ldc + col0, z, (int)imin64(32, p.N - col0));
+        for (int i = 0; i < NP; ++i) z[i] = make_uint4(0, 0, 0, 0);
+        for (int c = 0; c < BN / 32; ++c) {
+          const int64_t col0 = n0 + c * 32;
+          if (col0 >= p.N) break;
+          if (p.N - col0 >= 32) {
+            __syncwarp();
+            stage_put<RB>(stg, lane, z);
+            __syncwarp();
+            stage_store<RB>(stg, lane, c_rows + col0 * sizeof(TC), ldc_b, nrows);
+          } else if (vrow) {
+            float zf[32];
+#pragma unroll
+            for (int i = 0; i < 32; ++i) zf[i] = 0.f;
+            store_row32<TC>(Cb + grow * p.ldc + col0, zf, (int)(p.N - col0));
           }
         }
         continue;
       }
+      constexpr int NF = (EPI == 4) ? 8 : 4;  // 16-byte pieces per lane of one fetched block
+      const uint8_t* e_rows = (EPI == 4)
+          ? reinterpret_cast<const uint8_t*>(static_cast<const TC*>(p.h_in) + rbase * p.ldc)
+          : c_rows;
+      uint4 cur[NF], nxt[NF];
+      if (EPI == 2 || EPI == 4) epi_fetch<EPI>(e_rows, ldc_b, n0, lane, nrows, cur);
       if (!wait_bounded(smem_u32(&tfull[acc]), acc_phase, &s_abort, p.err)) break;
       tc_fence_after();
       const uint32_t tbase = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
       float v[32];
+      uint4 pk[NP];
       if (EPI == 3) {
-        // packed [gate 64 | up 64] blocks: a = silu(g) * u
+        // packed [gate 64 | up 64] blocks: h = [g | u] stored as computed, a = silu(g) * u
+        uint8_t* a_rows = reinterpret_cast<uint8_t*>(static_cast<TC*>(p.aux) + rbase * (p.N / 2));
+        const int64_t lda_b = (p.N / 2) * (int64_t)sizeof(TC);
         for (int blk = 0; blk < BN / 128; ++blk) {
           const int64_t cb = n0 + blk * 128;
           if (cb >= p.N) break;
 #pragma unroll 1
           for (int half = 0; half < 2; ++half) {
-            float u[32];
+            float u[32], a[32];
             tmem_ld32(tbase + blk * 128 + half * 32, v);
             tmem_ld32(tbase + blk * 128 + 64 + half * 32, u);
-            if (vrow) {
-              TC* hrow = Cb + grow * p.ldc;
-              store_row32<TC>(hrow + cb + half * 32, v, 32);
-              store_row32<TC>(hrow + cb + 64 + half * 32, u, 32);
-              float a[32];
 #pragma unroll
-              for (int i = 0; i < 32; ++i) a[i] = silu_f(v[i]) * u[i];
-              TC* arow = static_cast<TC*>(p.aux) + grow * (p.N / 2);
-              store_row32<TC>(arow + cb / 2 + half * 32, a, 32);
-            }
+            for (int i = 0; i < 32; ++i) a[i] = silu_f(v[i]) * u[i];
+#pragma unroll
+            for (int i = 0; i < NP; ++i) pk[i] = pack16<TC>(v + i * Vec<TC>::N);
+            __syncwarp();
+            stage_put<RB>(stg, lane, pk);
+            __syncwarp();
+            stage_store<RB>(stg, lane, c_rows + (cb + half * 32) * sizeof(TC), ldc_b, nrows);
+#pragma unroll
+            for (int i = 0; i < NP; ++i) pk[i] = pack16<TC>(u + i * Vec<TC>::N);
+            __syncwarp();
+            stage_put<RB>(stg, lane, pk);
+            __syncwarp();
+            stage_store<RB>(stg, lane, c_rows + (cb + 64 + half * 32) * sizeof(TC), ldc_b, nrows);
+#pragma unroll
+            for (int i = 0; i < NP; ++i) pk[i] = pack16<TC>(a + i * Vec<TC>::N);
+            __syncwarp();
+            stage_put<RB>(stg, lane, pk);
+            __syncwarp();
+            stage_store<RB>(stg, lane, a_rows + (cb / 2 + half * 32) * sizeof(TC), lda_b, nrows);
           }
+        }
+      } else if (EPI == 2 || EPI == 4) {
+        // EPI 2 reads the 32 x 32 block of C it adds to; EPI 4 reads the gate
+        // and up columns of the saved h.  Chunk c + 1's block is fetched into
+        // registers while chunk c is processed (chunk 0's before the wait).
+        const int nch = (int)imin64(BN / 32, (p.N - n0) / 32);
+        for (int c = 0; c < nch; ++c) {
+          const int64_t col0 = n0 + c * 32;
+          if (c + 1 < nch) epi_fetch<EPI>(e_rows, ldc_b, col0 + 32, lane, nrows, nxt);
+          tmem_ld32(tbase + c * 32, v);
+          __syncwarp();
+          epi_put<EPI>(stg, lane, cur);
+          __syncwarp();
+          if (EPI == 2) {
+            stage_get<RB>(stg, lane, pk);
+            float o[32];
+#pragma unroll
+            for (int i = 0; i < NP; ++i) unpack16<TC>(pk[i], o + i * Vec<TC>::N);
+#pragma unroll
+            for (int i = 0; i < 32; ++i) o[i] += v[i];
+#pragma unroll
+            for (int i = 0; i < NP; ++i) pk[i] = pack16<TC>(o + i * Vec<TC>::N);
+            stage_put<RB>(stg, lane, pk);
+            __syncwarp();
+            stage_store<RB>(stg, lane, c_rows + col0 * sizeof(TC), ldc_b, nrows);
+          } else {
+            uint4 gu[8];
+            stage_get<128>(stg, lane, gu);
+            float g[32], u[32];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              unpack16<TC>(gu[i], g + i * 8);
+              unpack16<TC>(gu[4 + i], u + i * 8);
+            }
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+              const float sg = sigmoid_f(g[i]);
+              const float dg = v[i] * u[i] * sg * (1.0f + g[i] * (1.0f - sg));
+              const float du = v[i] * g[i] * sg;
+              g[i] = dg;
+              u[i] = du;
+            }
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              gu[i] = pack16<TC>(g + i * 8);
+              gu[4 + i] = pack16<TC>(u + i * 8);
+            }
+            stage_put<128>(stg, lane, gu);
+            __syncwarp();
+            epi_store_gu(stg, lane, c_rows, ldc_b, col0, nrows);
+          }
+#pragma unroll
+          for (int i = 0; i < NF; ++i) cur[i] = nxt[i];
         }
       } else {
 #pragma unroll 1
@@ -505,45 +693,29 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
           const int64_t col0 = n0 + c * 32;
           if (col0 >= p.N) break;
           tmem_ld32(tbase + c * 32, v);
-          if (!vrow) continue;
           const int nvalid = (int)imin64(32, p.N - col0);
-          TC* crow = Cb + grow * p.ldc;
-          if (EPI == 0) {
-            store_row32<TC>(crow + col0, v, nvalid);
-          } else if (EPI == 1) {
-            if (p.bias) {
+          if (EPI == 1 || nvalid < 32) {
+            // router logits (E columns, possibly ragged): direct row stores
+            if (!vrow) continue;
+            TC* crow = Cb + grow * p.ldc;
+            if (EPI == 1 && p.bias) {
 #pragma unroll
               for (int i = 0; i < 32; ++i)
                 if (i < nvalid) v[i] += p.bias[col0 + i];
             }
-            store_row32<TC>(crow + col0, v, nvalid);
-          } else if (EPI == 2) {
-            if (nvalid == 32) {
-              float o[32];
-              load_row32<TC>(crow + col0, o);
-#pragma unroll
-              for (int i = 0; i < 32; ++i) v[i] += o[i];
-            } else {
+            if (EPI == 2) {
 #pragma unroll
               for (int i = 0; i < 32; ++i)
                 if (i < nvalid) v[i] += to_f32<TC>(crow[col0 + i]);
             }
             store_row32<TC>(crow + col0, v, nvalid);
-          } else if (EPI == 4) {
-            // v = dA for features col0 .. col0 + 31; gate / up columns in the packed order
-            const int64_t cg = (col0 / 64) * 128 + (col0 % 64);
-            const TC* hrow = static_cast<const TC*>(p.h_in) + grow * p.ldc;
-            float g[32], u[32], dg[32], du[32];
-            load_row32<TC>(hrow + cg, g);
-            load_row32<TC>(hrow + cg + 64, u);
+          } else if (EPI == 0) {
 #pragma unroll
-            for (int i = 0; i < 32; ++i) {
-              const float sg = sigmoid_f(g[i]);
-              dg[i] = v[i] * u[i] * sg * (1.0f + g[i] * (1.0f - sg));
-              du[i] = v[i] * g[i] * sg;
-            }
-            store_row32<TC>(crow + cg, dg, 32);
-            store_row32<TC>(crow + cg + 64, du, 32);
+            for (int i = 0; i < NP; ++i) pk[i] = pack16<TC>(v + i * Vec<TC>::N);
+            __syncwarp();
+            stage_put<RB>(stg, lane, pk);
+            __syncwarp();
+            stage_store<RB>(stg, lane, c_rows + col0 * sizeof(TC), ldc_b, nrows);
           }
         }
       }

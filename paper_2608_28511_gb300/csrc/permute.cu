@@ -151,28 +151,42 @@ cudaError_t launch_permutation(const Ctx& c, const int32_t* idx, const float* pr
 
 // ---------------------------------------------------------------------------
 // Row movers: one warp per token, lanes stride over the row's 16-byte vectors.
+// KM is a compile-time bound on K (2, 4, 8 or 16) so the per-token row and
+// load arrays stay in registers without the register cost of the largest K.
 // ---------------------------------------------------------------------------
 
+template <int KM>
 __device__ __forceinline__ void load_rows(const int32_t* __restrict__ row_of_slot, int64_t t, int K,
-                                          int32_t (&rows)[kMaxK]) {
+                                          int32_t (&rows)[KM]) {
 #pragma unroll
-  for (int k = 0; k < kMaxK; ++k) rows[k] = (k < K) ? __ldg(row_of_slot + t * K + k) : 0;
+  for (int k = 0; k < KM; ++k) rows[k] = (k < K) ? __ldg(row_of_slot + t * K + k) : 0;
 }
 
+static inline int k_bound(int K) { return K <= 2 ? 2 : (K <= 4 ? 4 : (K <= 8 ? 8 : 16)); }
+
+#define MOE_DISPATCH_KM(K, CALL) \
+  switch (k_bound(K)) {          \
+    case 2: { constexpr int KM = 2; CALL; break; }  \
+    case 4: { constexpr int KM = 4; CALL; break; }  \
+    case 8: { constexpr int KM = 8; CALL; break; }  \
+    default: { constexpr int KM = 16; CALL; break; } \
+  }
+
 // Dispatch: each token's row is read once and written to its K rows.
+template <int KM>
 __global__ void __launch_bounds__(256) dispatch_rows_kernel(const uint4* __restrict__ x,
                                                             const int32_t* __restrict__ row_of_slot, int64_t T,
                                                             int K, int vpr, uint4* __restrict__ x_perm) {
   const int lane = threadIdx.x & 31;
   const int64_t t = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   if (t >= T) return;
-  int32_t rows[kMaxK];
-  load_rows(row_of_slot, t, K, rows);
+  int32_t rows[KM];
+  load_rows<KM>(row_of_slot, t, K, rows);
   const uint4* src = x + t * vpr;
   for (int v = lane; v < vpr; v += 32) {
     const uint4 val = ld_stream(src + v);
 #pragma unroll
-    for (int k = 0; k < kMaxK; ++k)
+    for (int k = 0; k < KM; ++k)
       if (k < K) st_stream(x_perm + (int64_t)rows[k] * vpr + v, val);
   }
 }
@@ -181,14 +195,16 @@ cudaError_t launch_dispatch_rows(const Ctx& c, const void* x, const int32_t* row
                                  int64_t row_bytes, void* x_perm) {
   if (T == 0) return cudaSuccess;
   const int warps = 8;
+  const unsigned grid = (unsigned)((T + warps - 1) / warps);
+  const int vpr = (int)(row_bytes / 16);
   KernelScope ks("dispatch_rows", c.stream);
-  dispatch_rows_kernel<<<(unsigned)((T + warps - 1) / warps), 32 * warps, 0, c.stream>>>(
-      (const uint4*)x, row_of_slot, T, K, (int)(row_bytes / 16), (uint4*)x_perm);
+  MOE_DISPATCH_KM(K, (dispatch_rows_kernel<KM><<<grid, 32 * warps, 0, c.stream>>>(
+                         (const uint4*)x, row_of_slot, T, K, vpr, (uint4*)x_perm)));
   return cudaGetLastError();
 }
 
 // Combine: y[t] = sum_k p_k Y_perm[row_k], fp32 accumulation, one rounding.
-template <typename T>
+template <typename T, int KM>
 __global__ void __launch_bounds__(256) combine_kernel(const uint4* __restrict__ y_perm,
                                                       const float* __restrict__ prob_perm,
                                                       const int32_t* __restrict__ row_of_slot, int64_t Tn, int K,
@@ -197,21 +213,21 @@ __global__ void __launch_bounds__(256) combine_kernel(const uint4* __restrict__ 
   const int lane = threadIdx.x & 31;
   const int64_t t = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   if (t >= Tn) return;
-  int32_t rows[kMaxK];
-  load_rows(row_of_slot, t, K, rows);
-  float p[kMaxK];
+  int32_t rows[KM];
+  load_rows<KM>(row_of_slot, t, K, rows);
+  float p[KM];
 #pragma unroll
-  for (int k = 0; k < kMaxK; ++k) p[k] = (k < K) ? __ldg(prob_perm + rows[k]) : 0.f;
+  for (int k = 0; k < KM; ++k) p[k] = (k < K) ? __ldg(prob_perm + rows[k]) : 0.f;
   for (int v = lane; v < vpr; v += 32) {
+    uint4 raw[KM];
+#pragma unroll
+    for (int k = 0; k < KM; ++k)
+      if (k < K) raw[k] = ld_stream(y_perm + (int64_t)rows[k] * vpr + v);
     float acc[NV];
 #pragma unroll
     for (int i = 0; i < NV; ++i) acc[i] = 0.f;
-    uint4 raw[kMaxK];
 #pragma unroll
-    for (int k = 0; k < kMaxK; ++k)
-      if (k < K) raw[k] = ld_stream(y_perm + (int64_t)rows[k] * vpr + v);
-#pragma unroll
-    for (int k = 0; k < kMaxK; ++k) {
+    for (int k = 0; k < KM; ++k) {
       if (k < K) {
         float f[NV];
         unpack16<T>(raw[k], f);
@@ -230,17 +246,18 @@ cudaError_t launch_combine(const Ctx& c, DType dt, const void* y_perm, const flo
   const int vpr = (int)((int64_t)D * dsize(dt) / 16);
   const unsigned grid = (unsigned)((T + warps - 1) / warps);
   KernelScope ks("combine", c.stream);
-  if (dt == DType::BF16)
-    combine_kernel<bf16><<<grid, 32 * warps, 0, c.stream>>>((const uint4*)y_perm, prob_perm, row_of_slot, T, K,
-                                                            vpr, (uint4*)y);
-  else
-    combine_kernel<float><<<grid, 32 * warps, 0, c.stream>>>((const uint4*)y_perm, prob_perm, row_of_slot, T, K,
-                                                             vpr, (uint4*)y);
+  if (dt == DType::BF16) {
+    MOE_DISPATCH_KM(K, (combine_kernel<bf16, KM><<<grid, 32 * warps, 0, c.stream>>>(
+                           (const uint4*)y_perm, prob_perm, row_of_slot, T, K, vpr, (uint4*)y)));
+  } else {
+    MOE_DISPATCH_KM(K, (combine_kernel<float, KM><<<grid, 32 * warps, 0, c.stream>>>(
+                           (const uint4*)y_perm, prob_perm, row_of_slot, T, K, vpr, (uint4*)y)));
+  }
   return cudaGetLastError();
 }
 
 // Combine backward: dY_perm[row_k] = p_k dy[t]; dprob_perm[row_k] = <dy[t], Y_perm[row_k]>.
-template <typename T>
+template <typename T, int KM>
 __global__ void __launch_bounds__(256) combine_bwd_kernel(const uint4* __restrict__ dy,
                                                           const uint4* __restrict__ y_perm,
                                                           const float* __restrict__ prob_perm,
@@ -251,23 +268,24 @@ __global__ void __launch_bounds__(256) combine_bwd_kernel(const uint4* __restric
   const int lane = threadIdx.x & 31;
   const int64_t t = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   if (t >= Tn) return;
-  int32_t rows[kMaxK];
-  load_rows(row_of_slot, t, K, rows);
-  float p[kMaxK], dot[kMaxK];
+  int32_t rows[KM];
+  load_rows<KM>(row_of_slot, t, K, rows);
+  float p[KM], dot[KM];
 #pragma unroll
-  for (int k = 0; k < kMaxK; ++k) {
+  for (int k = 0; k < KM; ++k) {
     p[k] = (k < K) ? __ldg(prob_perm + rows[k]) : 0.f;
     dot[k] = 0.f;
   }
   for (int v = lane; v < vpr; v += 32) {
-    float g[NV];
-    unpack16<T>(ld_stream(dy + t * vpr + v), g);
-    uint4 raw[kMaxK];
+    const uint4 gv = ld_stream(dy + t * vpr + v);
+    uint4 raw[KM];
 #pragma unroll
-    for (int k = 0; k < kMaxK; ++k)
+    for (int k = 0; k < KM; ++k)
       if (k < K) raw[k] = ld_stream(y_perm + (int64_t)rows[k] * vpr + v);
+    float g[NV];
+    unpack16<T>(gv, g);
 #pragma unroll
-    for (int k = 0; k < kMaxK; ++k) {
+    for (int k = 0; k < KM; ++k) {
       if (k < K) {
         float f[NV], o[NV];
         unpack16<T>(raw[k], f);
@@ -281,7 +299,7 @@ __global__ void __launch_bounds__(256) combine_bwd_kernel(const uint4* __restric
     }
   }
 #pragma unroll
-  for (int k = 0; k < kMaxK; ++k) {
+  for (int k = 0; k < KM; ++k) {
     if (k < K) {
       float s = dot[k];
 #pragma unroll
@@ -299,20 +317,21 @@ cudaError_t launch_combine_bwd(const Ctx& c, DType dt, const void* dy, const voi
   const int vpr = (int)((int64_t)D * dsize(dt) / 16);
   const unsigned grid = (unsigned)((T + warps - 1) / warps);
   KernelScope ks("combine_bwd", c.stream);
-  if (dt == DType::BF16)
-    combine_bwd_kernel<bf16><<<grid, 32 * warps, 0, c.stream>>>((const uint4*)dy, (const uint4*)y_perm, prob_perm,
-                                                                row_of_slot, T, K, vpr, (uint4*)dy_perm,
-                                                                dprob_perm);
-  else
-    combine_bwd_kernel<float><<<grid, 32 * warps, 0, c.stream>>>((const uint4*)dy, (const uint4*)y_perm,
-                                                                 prob_perm, row_of_slot, T, K, vpr,
-                                                                 (uint4*)dy_perm, dprob_perm);
+  if (dt == DType::BF16) {
+    MOE_DISPATCH_KM(K, (combine_bwd_kernel<bf16, KM><<<grid, 32 * warps, 0, c.stream>>>(
+                           (const uint4*)dy, (const uint4*)y_perm, prob_perm, row_of_slot, T, K, vpr,
+                           (uint4*)dy_perm, dprob_perm)));
+  } else {
+    MOE_DISPATCH_KM(K, (combine_bwd_kernel<float, KM><<<grid, 32 * warps, 0, c.stream>>>(
+                           (const uint4*)dy, (const uint4*)y_perm, prob_perm, row_of_slot, T, K, vpr,
+                           (uint4*)dy_perm, dprob_perm)));
+  }
   return cudaGetLastError();
 }
 
 // Dispatch backward: dx[t] = sum_k dX_perm[row_k] (fp32 accumulation);
 // dprob[t, k] = dprob_perm[row_k].
-template <typename T>
+template <typename T, int KM>
 __global__ void __launch_bounds__(256) dispatch_bwd_kernel(const uint4* __restrict__ dx_perm,
                                                            const float* __restrict__ dprob_perm,
                                                            const int32_t* __restrict__ row_of_slot, int64_t Tn,
@@ -322,19 +341,19 @@ __global__ void __launch_bounds__(256) dispatch_bwd_kernel(const uint4* __restri
   const int lane = threadIdx.x & 31;
   const int64_t t = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   if (t >= Tn) return;
-  int32_t rows[kMaxK];
-  load_rows(row_of_slot, t, K, rows);
+  int32_t rows[KM];
+  load_rows<KM>(row_of_slot, t, K, rows);
   if (lane < K) dprob[t * K + lane] = __ldg(dprob_perm + row_of_slot[t * K + lane]);
   for (int v = lane; v < vpr; v += 32) {
+    uint4 raw[KM];
+#pragma unroll
+    for (int k = 0; k < KM; ++k)
+      if (k < K) raw[k] = ld_stream(dx_perm + (int64_t)rows[k] * vpr + v);
     float acc[NV];
 #pragma unroll
     for (int i = 0; i < NV; ++i) acc[i] = 0.f;
-    uint4 raw[kMaxK];
 #pragma unroll
-    for (int k = 0; k < kMaxK; ++k)
-      if (k < K) raw[k] = ld_stream(dx_perm + (int64_t)rows[k] * vpr + v);
-#pragma unroll
-    for (int k = 0; k < kMaxK; ++k) {
+    for (int k = 0; k < KM; ++k) {
       if (k < K) {
         float f[NV];
         unpack16<T>(raw[k], f);
@@ -353,12 +372,13 @@ cudaError_t launch_dispatch_bwd(const Ctx& c, DType dt, const void* dx_perm, con
   const int vpr = (int)((int64_t)D * dsize(dt) / 16);
   const unsigned grid = (unsigned)((T + warps - 1) / warps);
   KernelScope ks("dispatch_bwd", c.stream);
-  if (dt == DType::BF16)
-    dispatch_bwd_kernel<bf16><<<grid, 32 * warps, 0, c.stream>>>((const uint4*)dx_perm, dprob_perm, row_of_slot,
-                                                                 T, K, vpr, (uint4*)dx, dprob);
-  else
-    dispatch_bwd_kernel<float><<<grid, 32 * warps, 0, c.stream>>>((const uint4*)dx_perm, dprob_perm, row_of_slot,
-                                                                  T, K, vpr, (uint4*)dx, dprob);
+  if (dt == DType::BF16) {
+    MOE_DISPATCH_KM(K, (dispatch_bwd_kernel<bf16, KM><<<grid, 32 * warps, 0, c.stream>>>(
+                           (const uint4*)dx_perm, dprob_perm, row_of_slot, T, K, vpr, (uint4*)dx, dprob)));
+  } else {
+    MOE_DISPATCH_KM(K, (dispatch_bwd_kernel<float, KM><<<grid, 32 * warps, 0, c.stream>>>(
+                           (const uint4*)dx_perm, dprob_perm, row_of_slot, T, K, vpr, (uint4*)dx, dprob)));
+  }
   return cudaGetLastError();
 }
 
