@@ -50,7 +50,7 @@ def kernel_work(name: str, w: synth.Workload, T: int) -> tuple[str, float]:
     Din = w.H if w.H else D
     base = name.rsplit("_", 1)[0] if name.endswith(("_tc", "_simt")) else name
     flops = {
-        "ffn1_swiglu": 4.0 * TK * D * F, "ffn2": 2.0 * TK * F * D, "ffn2_dgrad_swiglu": 2.0 * TK * D * F,
+        "ffn1_swiglu": 4.0 * TK * D * F, "ffn2": 2.0 * TK * F * D, "ffn2_dgrad": 2.0 * TK * D * F,
         "ffn2_wgrad": 2.0 * TK * D * F, "ffn1_dgrad": 4.0 * TK * F * D, "ffn1_wgrad": 4.0 * TK * F * D,
         "latent_fwd": 2.0 * T * w.H * D, "latent_dgrad": 2.0 * T * w.H * D, "latent_wgrad": 2.0 * T * w.H * D,
         "router_dgrad": 2.0 * T * Din * E, "router_wgrad": 2.0 * T * Din * E,
@@ -66,6 +66,7 @@ def kernel_work(name: str, w: synth.Workload, T: int) -> tuple[str, float]:
         "combine_bwd": (T + 2 * TK) * D * bx + 12 * TK,
         "dispatch_bwd": (TK + T) * D * bx + 8 * TK,
         "route_dz": T * K * 12 + T * E * 6,
+        "swiglu_bwd": 5.0 * TK * F * bx,
         "pack_w1": 0.0,
     }
     return "hbm", float(byts.get(base, 0.0))
@@ -375,7 +376,7 @@ def main() -> None:
         roof = {"kernel": tname, "bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                 "frac": achieved / peak, "traffic": traffic, "peak_note": f"HBM copy, of {peaks['source']}"}
 
-    exp_ms = sum(v["ms_per_step"] for k, v in kernels.items() if k.startswith("ffn"))
+    exp_ms = sum(v["ms_per_step"] for k, v in kernels.items() if k.startswith("ffn") or k == "swiglu_bwd")
     perm_names = ("dispatch_rows", "combine", "combine_bwd", "dispatch_bwd")
     perm_ms = sum(v["ms_per_step"] for k, v in kernels.items() if k in perm_names)
     detail = {k: {"ms_per_step": round(v["ms_per_step"], 4),

@@ -170,7 +170,8 @@ size_t align_up(size_t v) { return (v + 255) & ~size_t(255); }
 // Workspace carve-up.  Calls are ordered on one stream, so the regions used by
 // different calls may overlap.
 size_t ws_perm(const Dims& d) { return align_up(perm_workspace_bytes(d.TK, d.E)); }
-size_t ws_ffn_bwd(const Dims& d) { return align_up((size_t)d.TK * 2 * d.F * d.bx); }
+// dH [TK, 2F] followed by dA [TK, F]
+size_t ws_ffn_bwd(const Dims& d) { return align_up((size_t)d.TK * 3 * d.F * d.bx); }
 size_t ws_route_bwd(const Dims& d) { return align_up((size_t)d.T * d.E * 2); }
 size_t ws_total(const Dims& d) {
   size_t m = ws_perm(d);
@@ -468,10 +469,11 @@ int moe_expert_ffn_bwd(const moe_shape_t* shape, const void* dy_perm, const void
   Ctx c;
   TRY(get_ctx(stream, &c));
   void* dH = ws;
-  // dgrad-2 with the SwiGLU backward epilogue: dA = dy_perm . w2_e -> dH
+  void* dA = static_cast<char*>(ws) + (size_t)d.TK * 2 * d.F * d.bx;
+  // dgrad-2: dA = dy_perm . w2_e, then the SwiGLU backward dA, h -> dH
   GemmDesc a;
   a.group = Group::M;
-  a.epi = Epi::SwigluBwd;
+  a.epi = Epi::Store;
   a.N = d.F;
   a.K = d.D;
   a.num_groups = d.E;
@@ -486,10 +488,9 @@ int moe_expert_ffn_bwd(const moe_shape_t* shape, const void* dy_perm, const void
   a.sb_n = 1;
   a.sb_k = d.F;
   a.sb_g = (int64_t)d.D * d.F;
-  a.C = dH;
+  a.C = dA;
   a.c_type = d.dt;
-  a.ldc = 2 * d.F;
-  a.h_in = h_save;
+  a.ldc = d.F;
   // wgrad-2: dw2_e[d, f] = sum_rows dy_perm[r, d] a[r, f]
   GemmDesc b;
   b.group = Group::K;
@@ -553,7 +554,10 @@ int moe_expert_ffn_bwd(const moe_shape_t* shape, const void* dy_perm, const void
   w.c_type = DType::F32;
   w.ldc = d.D;
   w.sc_g = (int64_t)2 * d.F * d.D;
-  if (d.TK > 0) TRY_CUDA(gemm(c, a, "ffn2_dgrad_swiglu_tc", "ffn2_dgrad_swiglu_simt"));
+  if (d.TK > 0) {
+    TRY_CUDA(gemm(c, a, "ffn2_dgrad_tc", "ffn2_dgrad_simt"));
+    TRY_CUDA(launch_swiglu_bwd(c, d.dt, dA, h_save, d.TK, d.F, dH));
+  }
   TRY_CUDA(gemm(c, b, "ffn2_wgrad_tc", "ffn2_wgrad_simt"));
   if (d.TK > 0) TRY_CUDA(gemm(c, cg, "ffn1_dgrad_tc", "ffn1_dgrad_simt"));
   TRY_CUDA(gemm(c, w, "ffn1_wgrad_tc", "ffn1_wgrad_simt"));

@@ -22,7 +22,6 @@ __device__ __forceinline__ float ldf(const void* p, int64_t i) {
 }
 
 __device__ __forceinline__ float silu_f(float v) { return v / (1.0f + __expf(-v)); }
-__device__ __forceinline__ float sigmoid_f(float v) { return 1.0f / (1.0f + __expf(-v)); }
 
 template <typename TA, typename TB, typename TC>
 __global__ void __launch_bounds__(256) simt_gemm_kernel(GemmDesc d) {
@@ -136,16 +135,6 @@ __global__ void __launch_bounds__(256) simt_gemm_kernel(GemmDesc d) {
             const int64_t f = n0 / 2 + col;
             static_cast<TC*>(d.aux)[gm * (d.N / 2) + f] = from_f32<TC>(silu_f(gt) * up);
           }
-          break;
-        }
-        case Epi::SwigluBwd: {
-          // gn is the feature f; its gate / up columns in the packed order
-          const int64_t cg = (gn / 64) * 128 + (gn % 64);
-          const TC* hrow = static_cast<const TC*>(d.h_in) + gm * d.ldc;
-          const float gt = to_f32<TC>(hrow[cg]), up = to_f32<TC>(hrow[cg + 64]);
-          const float sg = sigmoid_f(gt);
-          crow[cg] = from_f32<TC>(v * up * sg * (1.0f + gt * (1.0f - sg)));
-          crow[cg + 64] = from_f32<TC>(v * gt * sg);
           break;
         }
       }

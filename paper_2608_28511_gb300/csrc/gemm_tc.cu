@@ -79,9 +79,6 @@ bool make_plan(const GemmDesc& d, Plan* pl) {
     case Epi::SwigluFwd:
       if (d.c_type != DType::BF16 || d.N % 128 || !d.aux || !al16(d.aux)) return false;
       break;
-    case Epi::SwigluBwd:
-      if (d.c_type != DType::BF16 || d.N % 64 || !d.h_in || !al16(d.h_in)) return false;
-      break;
   }
   pl->bn = 256;
   if (d.group == Group::Dense && d.epi == Epi::StoreBias) pl->bn = d.N <= 64 ? 64 : (d.N <= 128 ? 128 : 256);
@@ -111,7 +108,6 @@ bool gemm_tc_supports(const GemmDesc& d) {
   // the instantiated combinations
   if (g == 1 && !pl.a_mn && !pl.b_mn && e == 3 && !f32) return true;
   if (g == 1 && !pl.a_mn && !pl.b_mn && e == 0 && !f32) return true;
-  if (g == 1 && !pl.a_mn && pl.b_mn && e == 4 && !f32) return true;
   if (g == 1 && !pl.a_mn && pl.b_mn && e == 0 && !f32) return true;
   if (g == 2 && pl.a_mn && pl.b_mn && e == 0 && f32) return true;
   if (g == 0 && !pl.a_mn && !pl.b_mn && e == 1 && f32) return true;
@@ -150,7 +146,6 @@ cudaError_t launch_gemm_tc(const Ctx& c, const GemmDesc& d, const char* name) {
   p.ldc = d.ldc;
   p.sc_g = d.sc_g;
   p.bias = d.bias;
-  p.h_in = d.h_in;
   p.aux = d.aux;
   p.err = c.err;
   int64_t ub;
@@ -164,7 +159,6 @@ cudaError_t launch_gemm_tc(const Ctx& c, const GemmDesc& d, const char* name) {
   KernelScope ks(name, c.stream);
   if (g == 1 && !pl.b_mn && e == 3) return launch_inst<256, false, false, 1, 3, bf16>(c, p, grid);
   if (g == 1 && !pl.b_mn && e == 0) return launch_inst<256, false, false, 1, 0, bf16>(c, p, grid);
-  if (g == 1 && pl.b_mn && e == 4) return launch_inst<256, false, true, 1, 4, bf16>(c, p, grid);
   if (g == 1 && pl.b_mn && e == 0) return launch_inst<256, false, true, 1, 0, bf16>(c, p, grid);
   if (g == 2) return launch_inst<256, true, true, 2, 0, float>(c, p, grid);
   if (g == 0 && e == 1) {

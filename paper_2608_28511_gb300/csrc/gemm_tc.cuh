@@ -44,7 +44,6 @@ struct Params {
   void* C;
   int64_t ldc, sc_g;
   const float* bias;
-  const void* h_in;
   void* aux;
   uint32_t* err;
 };
@@ -236,57 +235,23 @@ __device__ __forceinline__ void stage_store(const uint8_t* buf, int lane, uint8_
     if (r < nrows) *reinterpret_cast<uint4*>(gbase + r * ld_bytes + c * 16) = v;
   }
 }
-// Pieces of the 32-row block an EPI 2 / EPI 4 chunk reads, fetched into
-// registers (16 bytes per piece, rows >= nrows as zero).  EPI 2: 32 bf16
-// columns of C at col0 (4 pieces per lane).  EPI 4: the gate columns
-// cg .. cg+31 and up columns cg+64 .. cg+95 of h for features col0 .. col0+31
-// (8 pieces per lane; a staging row holds gate bytes 0..63, up bytes 64..127).
-template <int EPI>
-__device__ __forceinline__ void epi_fetch(const uint8_t* rows, int64_t ld_b, int64_t col0, int lane, int nrows,
+// The 32 x 32 bf16 block of C an accumulating chunk adds to, fetched into
+// registers as 16-byte pieces (4 per lane; rows >= nrows as zero), and put
+// into the staging buffer in row order.
+__device__ __forceinline__ void acc_fetch(const uint8_t* rows, int64_t ld_b, int64_t col0, int lane, int nrows,
                                           uint4* dst) {
-  if (EPI == 4) {
-    const int64_t cg = (col0 / 64) * 128 + (col0 % 64);
 #pragma unroll
-    for (int it = 0; it < 8; ++it) {
-      const int r = it * 4 + lane / 8, pc = lane % 8;
-      const int64_t off = pc < 4 ? cg * 2 + pc * 16 : (cg + 64) * 2 + (pc - 4) * 16;
-      dst[it] = r < nrows ? *reinterpret_cast<const uint4*>(rows + r * ld_b + off) : make_uint4(0, 0, 0, 0);
-    }
-  } else {
-#pragma unroll
-    for (int it = 0; it < 4; ++it) {
-      const int r = it * 8 + lane / 4, pc = lane % 4;
-      dst[it] = r < nrows ? *reinterpret_cast<const uint4*>(rows + r * ld_b + col0 * 2 + pc * 16)
-                          : make_uint4(0, 0, 0, 0);
-    }
+  for (int it = 0; it < 4; ++it) {
+    const int r = it * 8 + lane / 4, pc = lane % 4;
+    dst[it] = r < nrows ? *reinterpret_cast<const uint4*>(rows + r * ld_b + col0 * 2 + pc * 16)
+                        : make_uint4(0, 0, 0, 0);
   }
 }
-template <int EPI>
-__device__ __forceinline__ void epi_put(uint8_t* buf, int lane, const uint4* src) {
-  if (EPI == 4) {
+__device__ __forceinline__ void acc_put(uint8_t* buf, int lane, const uint4* src) {
 #pragma unroll
-    for (int it = 0; it < 8; ++it) {
-      const int r = it * 4 + lane / 8, pc = lane % 8;
-      *reinterpret_cast<uint4*>(buf + r * 144 + pc * 16) = src[it];
-    }
-  } else {
-#pragma unroll
-    for (int it = 0; it < 4; ++it) {
-      const int r = it * 8 + lane / 4, pc = lane % 4;
-      *reinterpret_cast<uint4*>(buf + r * 144 + pc * 16) = src[it];
-    }
-  }
-}
-// Staging rows [dg 64 B | du 64 B] -> dH gate and up columns of features col0 .. col0+31.
-__device__ __forceinline__ void epi_store_gu(const uint8_t* buf, int lane, uint8_t* rows, int64_t ld_b,
-                                             int64_t col0, int nrows) {
-  const int64_t cg = (col0 / 64) * 128 + (col0 % 64);
-#pragma unroll
-  for (int it = 0; it < 8; ++it) {
-    const int r = it * 4 + lane / 8, pc = lane % 8;
-    const int64_t off = pc < 4 ? cg * 2 + pc * 16 : (cg + 64) * 2 + (pc - 4) * 16;
-    const uint4 v = *reinterpret_cast<const uint4*>(buf + r * 144 + pc * 16);
-    if (r < nrows) *reinterpret_cast<uint4*>(rows + r * ld_b + off) = v;
+  for (int it = 0; it < 4; ++it) {
+    const int r = it * 8 + lane / 4, pc = lane % 4;
+    *reinterpret_cast<uint4*>(buf + r * 144 + pc * 16) = src[it];
   }
 }
 // gbase + r * ld_bytes -> buf rows 0..31 (rows r >= nrows read as zero).
@@ -373,7 +338,7 @@ __device__ __forceinline__ void load_row32(const T* src, float* v) {
   for (int i = 0; i < 32; i += NV) unpack16<T>(*reinterpret_cast<const uint4*>(src + i), v + i);
 }
 
-// EPI: 0 Store, 1 StoreBias, 2 Accum, 3 SwigluFwd, 4 SwigluBwd (values of moe::Epi).
+// EPI: 0 Store, 1 StoreBias, 2 Accum, 3 SwigluFwd (values of moe::Epi).
 template <int BN, bool A_MN, bool B_MN, int GROUP, int EPI, typename TC>
 __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_constant__ Params p) {
   using C = Cfg<BN>;
@@ -589,12 +554,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
         }
         continue;
       }
-      constexpr int NF = (EPI == 4) ? 8 : 4;  // 16-byte pieces per lane of one fetched block
-      const uint8_t* e_rows = (EPI == 4)
-          ? reinterpret_cast<const uint8_t*>(static_cast<const TC*>(p.h_in) + rbase * p.ldc)
-          : c_rows;
-      uint4 cur[NF], nxt[NF];
-      if (EPI == 2 || EPI == 4) epi_fetch<EPI>(e_rows, ldc_b, n0, lane, nrows, cur);
+      uint4 cur[4], nxt[4];  // an accumulating chunk's C block, fetched one chunk ahead
+      if (EPI == 2) acc_fetch(c_rows, ldc_b, n0, lane, nrows, cur);
       if (!wait_bounded(smem_u32(&tfull[acc]), acc_phase, &s_abort, p.err)) break;
       tc_fence_after();
       const uint32_t tbase = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
@@ -634,58 +595,30 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
             stage_store<RB>(stg, lane, a_rows + (cb / 2 + half * 32) * sizeof(TC), lda_b, nrows);
           }
         }
-      } else if (EPI == 2 || EPI == 4) {
-        // EPI 2 reads the 32 x 32 block of C it adds to; EPI 4 reads the gate
-        // and up columns of the saved h.  Chunk c + 1's block is fetched into
-        // registers while chunk c is processed (chunk 0's before the wait).
+      } else if (EPI == 2) {
+        // C += acc.  Chunk c + 1's C block is fetched into registers while
+        // chunk c is processed (chunk 0's before the accumulator wait).
         const int nch = (int)imin64(BN / 32, (p.N - n0) / 32);
         for (int c = 0; c < nch; ++c) {
           const int64_t col0 = n0 + c * 32;
-          if (c + 1 < nch) epi_fetch<EPI>(e_rows, ldc_b, col0 + 32, lane, nrows, nxt);
+          if (c + 1 < nch) acc_fetch(c_rows, ldc_b, col0 + 32, lane, nrows, nxt);
           tmem_ld32(tbase + c * 32, v);
           __syncwarp();
-          epi_put<EPI>(stg, lane, cur);
+          acc_put(stg, lane, cur);
           __syncwarp();
-          if (EPI == 2) {
-            stage_get<RB>(stg, lane, pk);
-            float o[32];
+          stage_get<RB>(stg, lane, pk);
+          float o[32];
 #pragma unroll
-            for (int i = 0; i < NP; ++i) unpack16<TC>(pk[i], o + i * Vec<TC>::N);
+          for (int i = 0; i < NP; ++i) unpack16<TC>(pk[i], o + i * Vec<TC>::N);
 #pragma unroll
-            for (int i = 0; i < 32; ++i) o[i] += v[i];
+          for (int i = 0; i < 32; ++i) o[i] += v[i];
 #pragma unroll
-            for (int i = 0; i < NP; ++i) pk[i] = pack16<TC>(o + i * Vec<TC>::N);
-            stage_put<RB>(stg, lane, pk);
-            __syncwarp();
-            stage_store<RB>(stg, lane, c_rows + col0 * sizeof(TC), ldc_b, nrows);
-          } else {
-            uint4 gu[8];
-            stage_get<128>(stg, lane, gu);
-            float g[32], u[32];
+          for (int i = 0; i < NP; ++i) pk[i] = pack16<TC>(o + i * Vec<TC>::N);
+          stage_put<RB>(stg, lane, pk);
+          __syncwarp();
+          stage_store<RB>(stg, lane, c_rows + col0 * sizeof(TC), ldc_b, nrows);
 #pragma unroll
-            for (int i = 0; i < 4; ++i) {
-              unpack16<TC>(gu[i], g + i * 8);
-              unpack16<TC>(gu[4 + i], u + i * 8);
-            }
-#pragma unroll
-            for (int i = 0; i < 32; ++i) {
-              const float sg = sigmoid_f(g[i]);
-              const float dg = v[i] * u[i] * sg * (1.0f + g[i] * (1.0f - sg));
-              const float du = v[i] * g[i] * sg;
-              g[i] = dg;
-              u[i] = du;
-            }
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-              gu[i] = pack16<TC>(g + i * 8);
-              gu[4 + i] = pack16<TC>(u + i * 8);
-            }
-            stage_put<128>(stg, lane, gu);
-            __syncwarp();
-            epi_store_gu(stg, lane, c_rows, ldc_b, col0, nrows);
-          }
-#pragma unroll
-          for (int i = 0; i < NF; ++i) cur[i] = nxt[i];
+          for (int i = 0; i < 4; ++i) cur[i] = nxt[i];
         }
       } else {
 #pragma unroll 1

@@ -74,6 +74,10 @@ cudaError_t launch_dispatch_bwd(const Ctx& c, DType dt, const void* dx_perm, con
 cudaError_t launch_pack_w1(const Ctx& c, DType dt, const void* w_gate, const void* w_up, int E, int F, int D,
                            void* w1);
 
+// swiglu.cu: dH [rows, 2F] (packed) from dA [rows, F] and the saved h [rows, 2F].
+cudaError_t launch_swiglu_bwd(const Ctx& c, DType dt, const void* dA, const void* h, int64_t rows, int F,
+                              void* dH);
+
 // ---------------------------------------------------------------------------
 // Grouped GEMM  C(m, n) = sum_k A(m, k) B(n, k), fp32 accumulation.
 // ---------------------------------------------------------------------------
@@ -88,7 +92,6 @@ enum class Epi : int {
   StoreBias = 1,  // C = acc + bias[n]
   Accum = 2,      // C = C + acc
   SwigluFwd = 3,  // acc is h (packed gate/up, N = 2F): C = h, aux[m, f] = silu(g) u  (aux ld = N/2)
-  SwigluBwd = 4,  // acc is dA (N = F): reads h_in [m, 2F], writes C = dH [m, 2F] (ldc = 2F)
 };
 
 struct GemmDesc {
@@ -108,7 +111,6 @@ struct GemmDesc {
   DType c_type = DType::BF16;
   int64_t ldc = 0, sc_g = 0;
   const float* bias = nullptr;       // StoreBias
-  const void* h_in = nullptr;        // SwigluBwd (c_type)
   void* aux = nullptr;               // SwigluFwd activation output (c_type)
 };
 
