@@ -51,6 +51,7 @@ bool al16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
 
 struct Plan {
   int bn;
+  int cg;  // CTAs per tile: 2 (a cluster pair, 256-row tiles) or 1 (128-row tiles)
   bool a_mn, b_mn;
   int64_t lda, ldb;
 };
@@ -81,21 +82,75 @@ bool make_plan(const GemmDesc& d, Plan* pl) {
       break;
   }
   pl->bn = 256;
-  if (d.group == Group::Dense && d.epi == Epi::StoreBias) pl->bn = d.N <= 64 ? 64 : (d.N <= 128 ? 128 : 256);
+  pl->cg = 1;
+  if (d.group == Group::Dense && d.epi == Epi::StoreBias) {
+    pl->bn = d.N <= 64 ? 64 : (d.N <= 128 ? 128 : 256);  // router logits: N = E
+  } else if (d.group == Group::M || (d.group == Group::Dense && d.M > BM)) {
+    pl->cg = 2;
+  }
   return true;
 }
 
-template <int BN, bool A_MN, bool B_MN, int GROUP, int EPI, typename TC>
-cudaError_t launch_inst(const Ctx& c, const Params& p, int grid) {
-  auto k = tc::gemm_tc_kernel<BN, A_MN, B_MN, GROUP, EPI, TC>;
+// Co-resident 2-CTA clusters of an instantiation (0 if the query fails).
+template <typename KernelT>
+int max_pair_clusters(KernelT k, int smem) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(2, 1, 1);
+  cfg.blockDim = dim3(tc::kThreads, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, k, &cfg) != cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
+  return n;
+}
+
+// ub = upper bound on the number of tiles (each tile is one CTA, or one pair for CG 2).
+template <int BN, bool A_MN, bool B_MN, int GROUP, int EPI, typename TC, int CG>
+cudaError_t launch_inst(const Ctx& c, const Params& p, int64_t ub) {
+  auto k = tc::gemm_tc_kernel<BN, A_MN, B_MN, GROUP, EPI, TC, CG>;
+  constexpr int kSmem = Cfg<BN, CG>::kSmem;
   static bool configured = false;
+  static int pairs = 0;
   if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg<BN>::kSmem);
+    cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmem);
     if (e != cudaSuccess) return e;
+    if (CG == 2) {
+      e = cudaFuncSetAttribute(k, cudaFuncAttributeNonPortableClusterSizeAllowed, 0);
+      (void)e;
+      cudaGetLastError();
+      pairs = max_pair_clusters(k, kSmem);
+    }
     configured = true;
   }
-  k<<<grid, tc::kThreads, Cfg<BN>::kSmem, c.stream>>>(p);
-  return cudaGetLastError();
+  if (CG == 1) {
+    const int grid = (int)(ub < c.num_sms ? ub : c.num_sms);
+    k<<<grid, tc::kThreads, kSmem, c.stream>>>(p);
+    return cudaGetLastError();
+  }
+  int np = pairs > 0 ? pairs : c.num_sms / 2;
+  if (ub < np) np = (int)ub;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(2 * np, 1, 1);
+  cfg.blockDim = dim3(tc::kThreads, 1, 1);
+  cfg.dynamicSmemBytes = kSmem;
+  cfg.stream = c.stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, k, p);
 }
 
 }  // namespace
@@ -122,24 +177,24 @@ cudaError_t launch_gemm_tc(const Ctx& c, const GemmDesc& d, const char* name) {
   if (!make_plan(d, &pl) || !gemm_tc_supports(d)) return cudaErrorNotSupported;
   Params p;
   memset(&p, 0, sizeof(p));
-  const int bn = pl.bn;
+  const int bn = pl.bn, bmp = BM * pl.cg, bnc = bn / pl.cg;
   // A: K-major box {64 k, 128 m}; MN-major box {64 m, 64 k}
   const int64_t a_rows = pl.a_mn ? (d.group == Group::K ? d.max_rows : d.K) : (d.group == Group::M ? d.max_rows : d.M);
   const int64_t a_inner = pl.a_mn ? d.M : d.K;
   if (!make_map(&p.ta, d.A, a_inner, a_rows, pl.lda * 2, 64, pl.a_mn ? 64 : BM)) return cudaErrorInvalidValue;
-  // B: K-major box {64 k, BN n}; MN-major box {64 n, 64 k}
+  // B: K-major box {64 k, BN / CG n}; MN-major box {64 n, 64 k}
   const int64_t grows = d.group == Group::M ? d.sb_g / pl.ldb : 0;
   int64_t b_rows;
   if (pl.b_mn) b_rows = d.group == Group::M ? grows * d.num_groups : (d.group == Group::K ? d.max_rows : d.K);
   else b_rows = d.group == Group::M ? grows * d.num_groups : d.N;
   const int64_t b_inner = pl.b_mn ? d.N : d.K;
-  if (!make_map(&p.tb, d.B, b_inner, b_rows, pl.ldb * 2, 64, pl.b_mn ? 64 : bn)) return cudaErrorInvalidValue;
+  if (!make_map(&p.tb, d.B, b_inner, b_rows, pl.ldb * 2, 64, pl.b_mn ? 64 : bnc)) return cudaErrorInvalidValue;
   p.M = d.M;
   p.N = d.N;
   p.K = d.K;
   p.b_group_rows = grows;
   p.num_groups = d.group == Group::Dense ? 1 : d.num_groups;
-  p.tiles_m = (int)((d.M + BM - 1) / BM);
+  p.tiles_m = (int)((d.M + bmp - 1) / bmp);
   p.tiles_n = (int)((d.N + bn - 1) / bn);
   p.offsets = d.offsets;
   p.C = d.C;
@@ -150,26 +205,31 @@ cudaError_t launch_gemm_tc(const Ctx& c, const GemmDesc& d, const char* name) {
   p.err = c.err;
   int64_t ub;
   if (d.group == Group::Dense) ub = (int64_t)p.tiles_m * p.tiles_n;
-  else if (d.group == Group::M) ub = ((d.max_rows + BM - 1) / BM + d.num_groups) * p.tiles_n;
+  else if (d.group == Group::M) ub = ((d.max_rows + bmp - 1) / bmp + d.num_groups) * p.tiles_n;
   else ub = (int64_t)d.num_groups * p.tiles_m * p.tiles_n;
   if (ub <= 0) return cudaSuccess;
-  const int grid = (int)(ub < c.num_sms ? ub : c.num_sms);
   const int g = (int)d.group, e = (int)d.epi;
-  const bool f32 = d.c_type == DType::F32;
   KernelScope ks(name, c.stream);
-  if (g == 1 && !pl.b_mn && e == 3) return launch_inst<256, false, false, 1, 3, bf16>(c, p, grid);
-  if (g == 1 && !pl.b_mn && e == 0) return launch_inst<256, false, false, 1, 0, bf16>(c, p, grid);
-  if (g == 1 && pl.b_mn && e == 0) return launch_inst<256, false, true, 1, 0, bf16>(c, p, grid);
-  if (g == 2) return launch_inst<256, true, true, 2, 0, float>(c, p, grid);
-  if (g == 0 && e == 1) {
-    if (bn == 64) return launch_inst<64, false, false, 0, 1, float>(c, p, grid);
-    if (bn == 128) return launch_inst<128, false, false, 0, 1, float>(c, p, grid);
-    return launch_inst<256, false, false, 0, 1, float>(c, p, grid);
+  if (pl.cg == 2) {
+    if (g == 1 && !pl.b_mn && e == 3) return launch_inst<256, false, false, 1, 3, bf16, 2>(c, p, ub);
+    if (g == 1 && !pl.b_mn && e == 0) return launch_inst<256, false, false, 1, 0, bf16, 2>(c, p, ub);
+    if (g == 1 && pl.b_mn && e == 0) return launch_inst<256, false, true, 1, 0, bf16, 2>(c, p, ub);
+    if (g == 0 && !pl.a_mn && !pl.b_mn && e == 0) return launch_inst<256, false, false, 0, 0, bf16, 2>(c, p, ub);
+    if (g == 0 && !pl.a_mn && pl.b_mn && e == 0) return launch_inst<256, false, true, 0, 0, bf16, 2>(c, p, ub);
+    if (g == 0 && !pl.a_mn && pl.b_mn && e == 2) return launch_inst<256, false, true, 0, 2, bf16, 2>(c, p, ub);
+    if (g == 0 && pl.a_mn && pl.b_mn) return launch_inst<256, true, true, 0, 0, float, 2>(c, p, ub);
+    return cudaErrorNotSupported;
   }
-  if (g == 0 && !pl.a_mn && !pl.b_mn && e == 0) return launch_inst<256, false, false, 0, 0, bf16>(c, p, grid);
-  if (g == 0 && !pl.a_mn && pl.b_mn && e == 0) return launch_inst<256, false, true, 0, 0, bf16>(c, p, grid);
-  if (g == 0 && !pl.a_mn && pl.b_mn && e == 2) return launch_inst<256, false, true, 0, 2, bf16>(c, p, grid);
-  if (g == 0 && pl.a_mn && pl.b_mn && f32) return launch_inst<256, true, true, 0, 0, float>(c, p, grid);
+  if (g == 2) return launch_inst<256, true, true, 2, 0, float, 1>(c, p, ub);
+  if (g == 0 && e == 1) {
+    if (bn == 64) return launch_inst<64, false, false, 0, 1, float, 1>(c, p, ub);
+    if (bn == 128) return launch_inst<128, false, false, 0, 1, float, 1>(c, p, ub);
+    return launch_inst<256, false, false, 0, 1, float, 1>(c, p, ub);
+  }
+  if (g == 0 && !pl.a_mn && !pl.b_mn && e == 0) return launch_inst<256, false, false, 0, 0, bf16, 1>(c, p, ub);
+  if (g == 0 && !pl.a_mn && pl.b_mn && e == 0) return launch_inst<256, false, true, 0, 0, bf16, 1>(c, p, ub);
+  if (g == 0 && !pl.a_mn && pl.b_mn && e == 2) return launch_inst<256, false, true, 0, 2, bf16, 1>(c, p, ub);
+  if (g == 0 && pl.a_mn && pl.b_mn) return launch_inst<256, true, true, 0, 0, float, 1>(c, p, ub);
   return cudaErrorNotSupported;
 }
 

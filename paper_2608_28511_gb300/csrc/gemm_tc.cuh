@@ -63,15 +63,26 @@ __device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
 __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
 }
+// CL: acquire at cluster scope (barriers that the other CTA of a pair signals).
+template <bool CL = false>
 __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
   uint32_t ok;
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-      "selp.u32 %0, 1, 0, p;\n\t}\n"
-      : "=r"(ok)
-      : "r"(bar), "r"(parity)
-      : "memory");
+  if (CL)
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}\n"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+  else
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}\n"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
   return ok != 0;
 }
 __device__ __forceinline__ uint64_t global_timer_ns() {
@@ -80,12 +91,13 @@ __device__ __forceinline__ uint64_t global_timer_ns() {
   return t;
 }
 // Wait for phase `parity` of `bar`; false if the CTA aborted or the limit expired.
+template <bool CL = false>
 __device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, volatile int* abort_flag,
                                              uint32_t* err) {
-  if (mbar_try_wait(bar, parity)) return true;
+  if (mbar_try_wait<CL>(bar, parity)) return true;
   const uint64_t t0 = global_timer_ns();
   for (uint32_t i = 1;; ++i) {
-    if (mbar_try_wait(bar, parity)) return true;
+    if (mbar_try_wait<CL>(bar, parity)) return true;
     if ((i & 63u) == 0) {
       if (*abort_flag) return false;
       if (global_timer_ns() - t0 > kWaitLimitNs) {
@@ -97,9 +109,10 @@ __device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, vola
   }
 }
 // Same, ignoring the abort flag (used while draining).
+template <bool CL = false>
 __device__ __forceinline__ bool wait_drain(uint32_t bar, uint32_t parity, uint64_t limit_ns) {
   const uint64_t t0 = global_timer_ns();
-  while (!mbar_try_wait(bar, parity)) {
+  while (!mbar_try_wait<CL>(bar, parity)) {
     if (global_timer_ns() - t0 > limit_ns) return false;
   }
   return true;
@@ -145,6 +158,82 @@ __device__ __forceinline__ void mma_commit(uint32_t bar) {
   asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
                : "memory");
 }
+// ---- CTA-pair (cta_group::2) forms: one leader CTA issues the MMAs of a
+// 256-row tile whose halves live in the two CTAs of a cluster of 2.
+__device__ __forceinline__ uint32_t cluster_ctarank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+// The shared::cluster address of `saddr`'s counterpart in CTA `rank` of the cluster.
+__device__ __forceinline__ uint32_t map_to_rank(uint32_t saddr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(saddr), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
+}
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+// TMA load into this CTA's shared memory that completes on an mbarrier of
+// either CTA of the pair (here: the leader's).
+__device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const CUtensorMap* map, uint32_t bar_cluster, int x,
+                                                 int y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%3, "
+      "%4}], [%2];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar_cluster), "r"(x), "r"(y)
+      : "memory");
+}
+template <int CG>
+__device__ __forceinline__ void tmem_alloc_cg(uint32_t dst_smem, uint32_t ncols) {
+  if (CG == 2)
+    asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem), "r"(ncols)
+                 : "memory");
+  else
+    tmem_alloc(dst_smem, ncols);
+}
+template <int CG>
+__device__ __forceinline__ void tmem_relinquish_cg() {
+  if (CG == 2) asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+  else tmem_relinquish();
+}
+template <int CG>
+__device__ __forceinline__ void tmem_dealloc_cg(uint32_t taddr, uint32_t ncols) {
+  if (CG == 2)
+    asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+  else
+    tmem_dealloc(taddr, ncols);
+}
+template <int CG>
+__device__ __forceinline__ void mma_bf16_cg(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                            uint32_t accumulate) {
+  if (CG == 2)
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}\n" ::"r"(d_tmem),
+        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+  else
+    mma_bf16(d_tmem, adesc, bdesc, idesc, accumulate);
+}
+// Arrive on `bar` (same offset) in every CTA of `mask` once this thread's
+// earlier MMAs complete.
+template <int CG>
+__device__ __forceinline__ void mma_commit_cg(uint32_t bar, uint16_t mask) {
+  if (CG == 2)
+    asm volatile(
+        "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
+            bar),
+        "h"(mask)
+        : "memory");
+  else
+    mma_commit(bar);
+}
+
 // 32 consecutive fp32 columns of this warp's 32 TMEM lanes (one row per thread).
 __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
   uint32_t r[32];
@@ -185,16 +274,21 @@ __device__ __forceinline__ uint64_t make_sdesc(uint32_t saddr, uint32_t lbo, uin
 }
 
 // Instruction descriptor for kind::f16: fp32 accumulator, bf16 A and B,
-// operand majorness, N >> 3 at bit 17, M >> 4 at bit 24.
-__host__ __device__ constexpr uint32_t make_idesc(int bn, bool a_mn, bool b_mn) {
+// operand majorness, N >> 3 at bit 17, M >> 4 at bit 24 (M = 128 per CTA,
+// 256 for a CTA pair).
+__host__ __device__ constexpr uint32_t make_idesc(int bn, int bm, bool a_mn, bool b_mn) {
   return (1u << 4) | (1u << 7) | (1u << 10) | ((a_mn ? 1u : 0u) << 15) | ((b_mn ? 1u : 0u) << 16) |
-         ((uint32_t)(bn >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
+         ((uint32_t)(bn >> 3) << 17) | ((uint32_t)(bm >> 4) << 24);
 }
 
-template <int BN>
+// CG = 1: one CTA computes a 128 x BN tile.  CG = 2: a cluster of two CTAs
+// computes a 256 x BN tile; each CTA stages its 128 rows of A and BN / 2 rows
+// of B, and holds its 128 accumulator rows in its own TMEM.
+template <int BN, int CG = 1>
 struct Cfg {
+  static constexpr int kBRows = BN / CG;
   static constexpr int kABytes = BM * BK * 2;
-  static constexpr int kBBytes = BN * BK * 2;
+  static constexpr int kBBytes = kBRows * BK * 2;
   static constexpr int kStageBytes = kABytes + kBBytes;
   static constexpr int kStages = (196608 / kStageBytes) < 8 ? (196608 / kStageBytes) : 8;
   static constexpr int kCols = 2 * BN;  // double-buffered fp32 accumulator
@@ -274,14 +368,16 @@ struct Tile {
   int nkb;
 };
 
-// Tile t of the static sequence.  GROUP: 0 dense, 1 by M, 2 by K.
-template <int GROUP>
+// Tile t of the static sequence.  GROUP: 0 dense, 1 by M, 2 by K.  Tiles
+// are BM * CG rows high; row0 is this CTA's first row (rank * BM into the tile).
+template <int GROUP, int CG = 1>
 __device__ __forceinline__ void decode_tile(const Params& p, int t, const int* s_off, const int* s_pref,
-                                            Tile& ti) {
+                                            uint32_t rank, Tile& ti) {
+  constexpr int BMP = BM * CG;
   if (GROUP == 0) {
     const int mt = t / p.tiles_n, nt = t % p.tiles_n;
     ti.g = 0;
-    ti.row0 = (int64_t)mt * BM;
+    ti.row0 = (int64_t)mt * BMP + rank * BM;
     ti.row_end = p.M;
     ti.n0 = nt;
     ti.kbeg = 0;
@@ -295,7 +391,7 @@ __device__ __forceinline__ void decode_tile(const Params& p, int t, const int* s
       else hi = mid - 1;
     }
     ti.g = lo;
-    ti.row0 = (int64_t)s_off[lo] + (int64_t)(mb - s_pref[lo]) * BM;
+    ti.row0 = (int64_t)s_off[lo] + (int64_t)(mb - s_pref[lo]) * BMP + rank * BM;
     ti.row_end = s_off[lo + 1];
     ti.n0 = nt;
     ti.kbeg = 0;
@@ -304,7 +400,7 @@ __device__ __forceinline__ void decode_tile(const Params& p, int t, const int* s
     const int per = p.tiles_m * p.tiles_n;
     const int g = t / per, rem = t % per;
     ti.g = g;
-    ti.row0 = (int64_t)(rem / p.tiles_n) * BM;
+    ti.row0 = (int64_t)(rem / p.tiles_n) * BMP + rank * BM;
     ti.row_end = p.M;
     ti.n0 = rem % p.tiles_n;
     ti.kbeg = s_off[g];
@@ -339,10 +435,16 @@ __device__ __forceinline__ void load_row32(const T* src, float* v) {
 }
 
 // EPI: 0 Store, 1 StoreBias, 2 Accum, 3 SwigluFwd (values of moe::Epi).
-template <int BN, bool A_MN, bool B_MN, int GROUP, int EPI, typename TC>
+// CG: 1 = one CTA per 128 x BN tile; 2 = a cluster of two CTAs per 256 x BN
+// tile (the even CTA issues the MMAs; both stage their halves and drain
+// their own accumulator rows).
+template <int BN, bool A_MN, bool B_MN, int GROUP, int EPI, typename TC, int CG>
 __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_constant__ Params p) {
-  using C = Cfg<BN>;
-  constexpr uint32_t kIdesc = make_idesc(BN, A_MN, B_MN);
+  using C = Cfg<BN, CG>;
+  constexpr int BMP = BM * CG;
+  constexpr int BNC = C::kBRows;
+  constexpr uint32_t kIdesc = make_idesc(BN, BMP, A_MN, B_MN);
+  static_assert(CG == 1 || GROUP != 2, "per-expert K grouping runs on single CTAs");
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::kStages * C::kStageBytes + C::kStagingBytes);
@@ -359,6 +461,9 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
 
   const int tid = threadIdx.x;
   const int warp = tid >> 5, lane = tid & 31;
+  const uint32_t rank = CG == 2 ? cluster_ctarank() : 0u;
+  const bool leader = rank == 0;
+  const int cta0 = blockIdx.x / CG, ncta = gridDim.x / CG;  // tile-walker index and count
 
   if (warp == 0 && lane == 0) {
     for (int s = 0; s < C::kStages; ++s) {
@@ -367,7 +472,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(smem_u32(&tfull[a]), 1);
-      mbar_init(smem_u32(&tempty[a]), 4);
+      mbar_init(smem_u32(&tempty[a]), 4 * CG);
     }
     mbar_init(smem_u32(done), 1);
     fence_barrier_init();
@@ -376,8 +481,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     tma_prefetch_desc(&p.tb);
   }
   if (warp == 1) {
-    tmem_alloc(smem_u32(s_tmem), C::kCols);
-    tmem_relinquish();
+    tmem_alloc_cg<CG>(smem_u32(s_tmem), C::kCols);
+    tmem_relinquish_cg<CG>();
   }
   if (GROUP != 0) {
     for (int i = tid; i <= p.num_groups; i += kThreads) s_off[i] = p.offsets[i];
@@ -390,7 +495,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
       int acc = 0;
       for (int g = 0; g < p.num_groups; ++g) {
         s_pref[g] = acc;
-        acc += (s_off[g + 1] - s_off[g] + BM - 1) / BM;
+        acc += (s_off[g + 1] - s_off[g] + BMP - 1) / BMP;
       }
       s_pref[p.num_groups] = acc;
       s_total = acc * p.tiles_n;
@@ -400,6 +505,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
   }
   tc_fence_before();
   __syncthreads();
+  if (CG == 2) cluster_sync();  // both CTAs' barriers exist before any cross-CTA signal
   tc_fence_after();
   const uint32_t tmem_base = *s_tmem;
   const int total = s_total;
@@ -412,60 +518,70 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
       int issued = 0;
       uint32_t last_phase = 0;  // bit s: phase of the last copy issued into stage s
       bool ok = true;
-      for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
+      for (int t = cta0; t < total && ok; t += ncta) {
         Tile ti;
-        decode_tile<GROUP>(p, t, s_off, s_pref, ti);
-        const int64_t n0 = ti.n0 * BN;
+        decode_tile<GROUP, CG>(p, t, s_off, s_pref, rank, ti);
+        const int64_t nb = ti.n0 * BN + (int64_t)rank * BNC;  // this CTA's first B row / column
         for (int kb = 0; kb < ti.nkb; ++kb) {
-          if (!wait_bounded(smem_u32(&empty[stage]), phase ^ 1u, &s_abort, p.err)) { ok = false; break; }
-          const uint32_t fb = smem_u32(&full[stage]);
-          mbar_expect_tx(fb, C::kStageBytes);
+          if (!wait_bounded<CG == 2>(smem_u32(&empty[stage]), phase ^ 1u, &s_abort, p.err)) { ok = false; break; }
+          const uint32_t fb_local = smem_u32(&full[stage]);
+          // CG 2: both CTAs' copies complete on the leader's barrier, which expects both
+          const uint32_t fb = CG == 2 ? map_to_rank(fb_local, 0) : fb_local;
+          if (leader) mbar_expect_tx(fb_local, CG * C::kStageBytes);
           const uint32_t sa = smem_u32(smem + stage * C::kStageBytes);
           const uint32_t sb = sa + C::kABytes;
           const int k0 = (int)(ti.kbeg + (int64_t)kb * BK);
+          auto load = [&](uint32_t dst, const CUtensorMap* m, int x, int y) {
+            if (CG == 2) tma_load_2d_pair(dst, m, fb, x, y);
+            else tma_load_2d(dst, m, fb, x, y);
+          };
           if (A_MN) {
-            tma_load_2d(sa, &p.ta, fb, (int)ti.row0, k0);
-            tma_load_2d(sa + 8192, &p.ta, fb, (int)ti.row0 + 64, k0);
+            load(sa, &p.ta, (int)ti.row0, k0);
+            load(sa + 8192, &p.ta, (int)ti.row0 + 64, k0);
           } else {
-            tma_load_2d(sa, &p.ta, fb, k0, (int)ti.row0);
+            load(sa, &p.ta, k0, (int)ti.row0);
           }
           if (B_MN) {
             const int ky = (int)(ti.g * p.b_group_rows) + k0;
 #pragma unroll
-            for (int j = 0; j < BN / 64; ++j) tma_load_2d(sb + j * 8192, &p.tb, fb, (int)n0 + 64 * j, ky);
+            for (int j = 0; j < BNC / 64; ++j) load(sb + j * 8192, &p.tb, (int)nb + 64 * j, ky);
           } else {
-            tma_load_2d(sb, &p.tb, fb, k0, (int)(ti.g * p.b_group_rows + n0));
+            load(sb, &p.tb, k0, (int)(ti.g * p.b_group_rows + nb));
           }
           last_phase = (last_phase & ~(1u << stage)) | (phase << stage);
           ++issued;
           if (++stage == C::kStages) { stage = 0; phase ^= 1u; }
         }
       }
-      // drain: every issued copy must land before the CTA exits
-      const int pending = issued < C::kStages ? issued : C::kStages;
-      for (int i = 0; i < pending; ++i) {
-        stage = (stage + C::kStages - 1) % C::kStages;
-        wait_drain(smem_u32(&full[stage]), (last_phase >> stage) & 1u, 1000000000ull);
+      // drain: every issued copy must land before the CTA exits (the leader's
+      // barriers also count the other CTA's copies)
+      if (leader) {
+        const int pending = issued < C::kStages ? issued : C::kStages;
+        for (int i = 0; i < pending; ++i) {
+          stage = (stage + C::kStages - 1) % C::kStages;
+          wait_drain<CG == 2>(smem_u32(&full[stage]), (last_phase >> stage) & 1u, 1000000000ull);
+        }
       }
     }
   } else if (warp == 1) {
-    // ------------------------------------------------------------ MMA issuer
+    // ------------------------------------------------------------ MMA issuer (the leader CTA)
     int stage = 0;
     uint32_t phase = 0;
     int acc = 0;
     uint32_t acc_phase = 0;
     bool ok = true;
     bool issued_any = false;
-    for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
+    constexpr uint16_t kBoth = 0x3;
+    for (int t = cta0; t < total && ok && leader; t += ncta) {
       Tile ti;
-      decode_tile<GROUP>(p, t, s_off, s_pref, ti);
+      decode_tile<GROUP, CG>(p, t, s_off, s_pref, rank, ti);
       if (ti.nkb == 0) continue;
       issued_any = true;
-      if (!wait_bounded(smem_u32(&tempty[acc]), acc_phase ^ 1u, &s_abort, p.err)) { ok = false; break; }
+      if (!wait_bounded<CG == 2>(smem_u32(&tempty[acc]), acc_phase ^ 1u, &s_abort, p.err)) { ok = false; break; }
       tc_fence_after();
       const uint32_t d_tmem = tmem_base + (uint32_t)(acc * BN);
       for (int kb = 0; kb < ti.nkb; ++kb) {
-        if (!wait_bounded(smem_u32(&full[stage]), phase, &s_abort, p.err)) { ok = false; break; }
+        if (!wait_bounded<CG == 2>(smem_u32(&full[stage]), phase, &s_abort, p.err)) { ok = false; break; }
         tc_fence_after();
         uint8_t* sa_ptr = smem + stage * C::kStageBytes;
         const uint32_t sa = smem_u32(sa_ptr);
@@ -495,22 +611,22 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
             else ad = make_sdesc(sa + k * 32, 16, 1024);
             if (B_MN) bd = make_sdesc(sb + k * 2048, 8192, 1024);
             else bd = make_sdesc(sb + k * 32, 16, 1024);
-            mma_bf16(d_tmem, ad, bd, kIdesc, (kb > 0 || k > 0) ? 1u : 0u);
+            mma_bf16_cg<CG>(d_tmem, ad, bd, kIdesc, (kb > 0 || k > 0) ? 1u : 0u);
           }
-          mma_commit(smem_u32(&empty[stage]));
+          mma_commit_cg<CG>(smem_u32(&empty[stage]), kBoth);
         }
         __syncwarp();
         if (++stage == C::kStages) { stage = 0; phase ^= 1u; }
       }
       if (!ok) break;
-      if (lane == 0) mma_commit(smem_u32(&tfull[acc]));
+      if (lane == 0) mma_commit_cg<CG>(smem_u32(&tfull[acc]), kBoth);
       __syncwarp();
       if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
     }
     // drain: all MMAs issued by this warp have completed before TMEM is freed
     if (lane == 0 && issued_any) {
-      mma_commit(smem_u32(done));
-      wait_drain(smem_u32(done), 0, 1000000000ull);
+      mma_commit_cg<CG>(smem_u32(done), 0x1);
+      wait_drain<CG == 2>(smem_u32(done), 0, 1000000000ull);
     }
     __syncwarp();
   } else {
@@ -522,9 +638,9 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     const int64_t ldc_b = p.ldc * (int64_t)sizeof(TC);
     int acc = 0;
     uint32_t acc_phase = 0;
-    for (int t = blockIdx.x; t < total; t += gridDim.x) {
+    for (int t = cta0; t < total; t += ncta) {
       Tile ti;
-      decode_tile<GROUP>(p, t, s_off, s_pref, ti);
+      decode_tile<GROUP, CG>(p, t, s_off, s_pref, rank, ti);
       const int64_t n0 = ti.n0 * BN;
       const int64_t rbase = ti.row0 + q * 32;  // this warp's first row
       const int nrows = (int)imax64(0, imin64(32, ti.row_end - rbase));
@@ -556,7 +672,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
       }
       uint4 cur[4], nxt[4];  // an accumulating chunk's C block, fetched one chunk ahead
       if (EPI == 2) acc_fetch(c_rows, ldc_b, n0, lane, nrows, cur);
-      if (!wait_bounded(smem_u32(&tfull[acc]), acc_phase, &s_abort, p.err)) break;
+      if (!wait_bounded<CG == 2>(smem_u32(&tfull[acc]), acc_phase, &s_abort, p.err)) break;
       tc_fence_after();
       const uint32_t tbase = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
       float v[32];
@@ -654,15 +770,20 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(smem_u32(&tempty[acc]));
+      if (lane == 0) {
+        // the accumulator buffer is free once every epilogue warp of the tile drained it
+        if (CG == 2) mbar_arrive_cluster(map_to_rank(smem_u32(&tempty[acc]), 0));
+        else mbar_arrive(smem_u32(&tempty[acc]));
+      }
       if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
     }
   }
 
   tc_fence_before();
   __syncthreads();
+  if (CG == 2) cluster_sync();  // neither CTA frees TMEM or exits while the other may still signal it
   tc_fence_after();
-  if (warp == 1) tmem_dealloc(tmem_base, C::kCols);
+  if (warp == 1) tmem_dealloc_cg<CG>(tmem_base, C::kCols);
 }
 
 }  // namespace tc
