@@ -170,8 +170,9 @@ size_t align_up(size_t v) { return (v + 255) & ~size_t(255); }
 // Workspace carve-up.  Calls are ordered on one stream, so the regions used by
 // different calls may overlap.
 size_t ws_perm(const Dims& d) { return align_up(perm_workspace_bytes(d.TK, d.E)); }
-// dH [TK, 2F] followed by dA [TK, F]
-size_t ws_ffn_bwd(const Dims& d) { return align_up((size_t)d.TK * 3 * d.F * d.bx); }
+// dH [TK, 2F], dA [TK, F], then the wgrad GEMMs' per-expert tensor maps
+size_t ws_ffn_bwd_maps_offset(const Dims& d) { return align_up((size_t)d.TK * 3 * d.F * d.bx); }
+size_t ws_ffn_bwd(const Dims& d) { return ws_ffn_bwd_maps_offset(d) + align_up(gemm_tc_group_scratch_bytes(d.E)); }
 size_t ws_route_bwd(const Dims& d) { return align_up((size_t)d.T * d.E * 2); }
 size_t ws_total(const Dims& d) {
   size_t m = ws_perm(d);
@@ -470,6 +471,7 @@ int moe_expert_ffn_bwd(const moe_shape_t* shape, const void* dy_perm, const void
   TRY(get_ctx(stream, &c));
   void* dH = ws;
   void* dA = static_cast<char*>(ws) + (size_t)d.TK * 2 * d.F * d.bx;
+  void* maps = static_cast<char*>(ws) + ws_ffn_bwd_maps_offset(d);
   // dgrad-2: dA = dy_perm . w2_e, then the SwiGLU backward dA, h -> dH
   GemmDesc a;
   a.group = Group::M;
@@ -508,6 +510,7 @@ int moe_expert_ffn_bwd(const moe_shape_t* shape, const void* dy_perm, const void
   b.sb_n = 1;
   b.sb_k = d.F;
   b.max_rows = d.TK;
+  b.scratch = maps;
   b.C = dw2;
   b.c_type = DType::F32;
   b.ldc = d.F;
@@ -550,6 +553,7 @@ int moe_expert_ffn_bwd(const moe_shape_t* shape, const void* dy_perm, const void
   w.sb_n = 1;
   w.sb_k = d.D;
   w.max_rows = d.TK;
+  w.scratch = maps;
   w.C = dw1;
   w.c_type = DType::F32;
   w.ldc = d.D;

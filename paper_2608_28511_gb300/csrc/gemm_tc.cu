@@ -68,6 +68,7 @@ bool make_plan(const GemmDesc& d, Plan* pl) {
   if ((pl->lda * 2) % 16 || (pl->ldb * 2) % 16) return false;
   if (!al16(d.A) || !al16(d.B) || !al16(d.C)) return false;
   if (d.group == Group::K && !(pl->a_mn && pl->b_mn)) return false;
+  if (d.group == Group::K && (!d.scratch || ((uintptr_t)d.scratch & 127u) || d.max_rows <= 0)) return false;
   if (d.group == Group::M && pl->a_mn) return false;
   if (d.group == Group::M && (d.sb_g % pl->ldb)) return false;
   if (d.group != Group::Dense && (d.num_groups <= 0 || d.num_groups > kMaxE || !d.offsets)) return false;
@@ -85,7 +86,7 @@ bool make_plan(const GemmDesc& d, Plan* pl) {
   pl->cg = 1;
   if (d.group == Group::Dense && d.epi == Epi::StoreBias) {
     pl->bn = d.N <= 64 ? 64 : (d.N <= 128 ? 128 : 256);  // router logits: N = E
-  } else if (d.group == Group::M || (d.group == Group::Dense && d.M > BM)) {
+  } else if (d.group == Group::M || d.M > BM) {
     pl->cg = 2;
   }
   return true;
@@ -155,6 +156,8 @@ cudaError_t launch_inst(const Ctx& c, const Params& p, int64_t ub) {
 
 }  // namespace
 
+size_t gemm_tc_group_scratch_bytes(int num_groups) { return (size_t)num_groups * 2 * sizeof(CUtensorMap); }
+
 bool gemm_tc_supports(const GemmDesc& d) {
   Plan pl;
   if (!make_plan(d, &pl)) return false;
@@ -209,8 +212,22 @@ cudaError_t launch_gemm_tc(const Ctx& c, const GemmDesc& d, const char* name) {
   else ub = (int64_t)d.num_groups * p.tiles_m * p.tiles_n;
   if (ub <= 0) return cudaSuccess;
   const int g = (int)d.group, e = (int)d.epi;
+  if (d.group == Group::K) {
+    // per-group maps: the templates above with the base and row extent moved per group
+    CUtensorMap* maps = static_cast<CUtensorMap*>(d.scratch);
+    {
+      KernelScope ks("group_maps", c.stream);
+      tc::build_group_maps<<<(d.num_groups + 127) / 128, 128, 0, c.stream>>>(
+          p.ta, p.tb, d.offsets, d.num_groups, static_cast<const uint8_t*>(d.A), pl.lda * 2,
+          static_cast<const uint8_t*>(d.B), pl.ldb * 2, maps);
+    }
+    cudaError_t st = cudaGetLastError();
+    if (st != cudaSuccess) return st;
+    p.gmaps = maps;
+  }
   KernelScope ks(name, c.stream);
   if (pl.cg == 2) {
+    if (g == 2) return launch_inst<256, true, true, 2, 0, float, 2>(c, p, ub);
     if (g == 1 && !pl.b_mn && e == 3) return launch_inst<256, false, false, 1, 3, bf16, 2>(c, p, ub);
     if (g == 1 && !pl.b_mn && e == 0) return launch_inst<256, false, false, 1, 0, bf16, 2>(c, p, ub);
     if (g == 1 && pl.b_mn && e == 0) return launch_inst<256, false, true, 1, 0, bf16, 2>(c, p, ub);

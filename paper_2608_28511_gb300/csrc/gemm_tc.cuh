@@ -13,8 +13,8 @@
 //
 // Grouping: Group::M tiles never mix experts in an output row range (rows
 // past an expert's end are computed and dropped); Group::K reduces each
-// expert over its own row range, zeroing the rows of the last partial k-block
-// that belong to the next expert before the MMA reads them.
+// expert over its own row range through per-expert tensor maps (built on the
+// device by build_group_maps), so the copy engine zero-fills past the end.
 //
 // Every mbarrier wait is bounded (kWaitLimitNs); on expiry the CTA sets the
 // device status word, drains its own copies and MMAs, frees TMEM and exits.
@@ -46,6 +46,7 @@ struct Params {
   const float* bias;
   void* aux;
   uint32_t* err;
+  const CUtensorMap* gmaps;  // Group::K: per group {A, B} maps whose rows start at the group's first row
 };
 
 // ---------------------------------------------------------------------------
@@ -126,6 +127,12 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map
 }
 __device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap* map) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
+}
+// A tensor map written in global memory by an earlier kernel: order its
+// generic-proxy writes before this thread's TMA reads of it.
+__device__ __forceinline__ void tmap_acquire(const CUtensorMap* map) {
+  asm volatile("fence.proxy.tensormap::generic.acquire.gpu [%0], 128;" ::"l"(reinterpret_cast<uint64_t>(map))
+               : "memory");
 }
 __device__ __forceinline__ void tmem_alloc(uint32_t dst_smem, uint32_t ncols) {
   asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem), "r"(ncols)
@@ -444,7 +451,6 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
   constexpr int BMP = BM * CG;
   constexpr int BNC = C::kBRows;
   constexpr uint32_t kIdesc = make_idesc(BN, BMP, A_MN, B_MN);
-  static_assert(CG == 1 || GROUP != 2, "per-expert K grouping runs on single CTAs");
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::kStages * C::kStageBytes + C::kStagingBytes);
@@ -517,6 +523,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
       uint32_t phase = 0;
       int issued = 0;
       uint32_t last_phase = 0;  // bit s: phase of the last copy issued into stage s
+      int cur_g = -1;           // group whose maps this thread has acquired (Group::K)
       bool ok = true;
       for (int t = cta0; t < total && ok; t += ncta) {
         Tile ti;
@@ -535,18 +542,36 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
             if (CG == 2) tma_load_2d_pair(dst, m, fb, x, y);
             else tma_load_2d(dst, m, fb, x, y);
           };
-          if (A_MN) {
-            load(sa, &p.ta, (int)ti.row0, k0);
-            load(sa + 8192, &p.ta, (int)ti.row0 + 64, k0);
-          } else {
-            load(sa, &p.ta, k0, (int)ti.row0);
-          }
-          if (B_MN) {
-            const int ky = (int)(ti.g * p.b_group_rows) + k0;
+          if (GROUP == 2) {
+            // the group's own maps: k rows count from the group's first row and
+            // the copy engine zero-fills rows past its end (the next group's rows
+            // never enter the reduction)
+            const CUtensorMap* ma = p.gmaps + 2 * ti.g;
+            const CUtensorMap* mb = ma + 1;
+            if (ti.g != cur_g) {
+              tmap_acquire(ma);
+              tmap_acquire(mb);
+              cur_g = ti.g;
+            }
+            const int ky = kb * BK;
+            load(sa, ma, (int)ti.row0, ky);
+            load(sa + 8192, ma, (int)ti.row0 + 64, ky);
 #pragma unroll
-            for (int j = 0; j < BNC / 64; ++j) load(sb + j * 8192, &p.tb, (int)nb + 64 * j, ky);
+            for (int j = 0; j < BNC / 64; ++j) load(sb + j * 8192, mb, (int)nb + 64 * j, ky);
           } else {
-            load(sb, &p.tb, k0, (int)(ti.g * p.b_group_rows + nb));
+            if (A_MN) {
+              load(sa, &p.ta, (int)ti.row0, k0);
+              load(sa + 8192, &p.ta, (int)ti.row0 + 64, k0);
+            } else {
+              load(sa, &p.ta, k0, (int)ti.row0);
+            }
+            if (B_MN) {
+              const int ky = (int)(ti.g * p.b_group_rows) + k0;
+#pragma unroll
+              for (int j = 0; j < BNC / 64; ++j) load(sb + j * 8192, &p.tb, (int)nb + 64 * j, ky);
+            } else {
+              load(sb, &p.tb, k0, (int)(ti.g * p.b_group_rows + nb));
+            }
           }
           last_phase = (last_phase & ~(1u << stage)) | (phase << stage);
           ++issued;
@@ -583,26 +608,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
       for (int kb = 0; kb < ti.nkb; ++kb) {
         if (!wait_bounded<CG == 2>(smem_u32(&full[stage]), phase, &s_abort, p.err)) { ok = false; break; }
         tc_fence_after();
-        uint8_t* sa_ptr = smem + stage * C::kStageBytes;
-        const uint32_t sa = smem_u32(sa_ptr);
+        const uint32_t sa = smem_u32(smem + stage * C::kStageBytes);
         const uint32_t sb = sa + C::kABytes;
-        if (GROUP == 2) {
-          // rows k >= kend of the last k-block belong to the next expert: zero them in A
-          const int64_t k0 = ti.kbeg + (int64_t)kb * BK;
-          const int valid = (int)imin64(BK, ti.kend - k0);
-          if (valid < BK) {
-            uint4 z = make_uint4(0, 0, 0, 0);
-            const int nrow = BK - valid;  // per chunk; 8 x 16 B per 128-byte row
-            for (int i = lane; i < 2 * nrow * 8; i += 32) {
-              const int chunk = i / (nrow * 8);
-              const int r = valid + (i % (nrow * 8)) / 8;
-              const int q = i % 8;
-              *reinterpret_cast<uint4*>(sa_ptr + chunk * 8192 + r * 128 + q * 16) = z;
-            }
-            fence_proxy_async_smem();
-          }
-          __syncwarp();
-        }
         if (lane == 0) {
 #pragma unroll
           for (int k = 0; k < BK / 16; ++k) {
@@ -784,6 +791,39 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
   if (CG == 2) cluster_sync();  // neither CTA frees TMEM or exits while the other may still signal it
   tc_fence_after();
   if (warp == 1) tmem_dealloc_cg<CG>(tmem_base, C::kCols);
+}
+
+// Per-group tensor maps for Group::K: group g's A and B maps are copies of
+// the full-tensor templates with the base moved to the group's first row and
+// the row extent set to the group's row count (at least 1), so a copy that
+// runs past the group's rows reads zeros.  out[2g] = A, out[2g + 1] = B.
+__global__ void build_group_maps(const __grid_constant__ CUtensorMap ta, const __grid_constant__ CUtensorMap tb,
+                                 const int32_t* __restrict__ offsets, int G, const uint8_t* a_base,
+                                 int64_t a_row_bytes, const uint8_t* b_base, int64_t b_row_bytes,
+                                 CUtensorMap* out) {
+  const int g = blockIdx.x * blockDim.x + threadIdx.x;
+  if (g >= G) return;
+  const int64_t lo = offsets[g];
+  const int64_t rows = offsets[g + 1] - lo;
+  const uint32_t dim = rows > 0 ? (uint32_t)rows : 1u;
+  CUtensorMap* ma = out + 2 * g;
+  CUtensorMap* mb = ma + 1;
+  const uint4* sa = reinterpret_cast<const uint4*>(&ta);
+  const uint4* sb = reinterpret_cast<const uint4*>(&tb);
+  uint4* da = reinterpret_cast<uint4*>(ma);
+  uint4* db = reinterpret_cast<uint4*>(mb);
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    da[i] = sa[i];
+    db[i] = sb[i];
+  }
+  const uint64_t pa = reinterpret_cast<uint64_t>(a_base + lo * a_row_bytes);
+  const uint64_t pb = reinterpret_cast<uint64_t>(b_base + lo * b_row_bytes);
+  asm volatile("tensormap.replace.tile.global_address.global.b1024.b64 [%0], %1;" ::"l"(ma), "l"(pa) : "memory");
+  asm volatile("tensormap.replace.tile.global_dim.global.b1024.b32 [%0], 1, %1;" ::"l"(ma), "r"(dim) : "memory");
+  asm volatile("tensormap.replace.tile.global_address.global.b1024.b64 [%0], %1;" ::"l"(mb), "l"(pb) : "memory");
+  asm volatile("tensormap.replace.tile.global_dim.global.b1024.b32 [%0], 1, %1;" ::"l"(mb), "r"(dim) : "memory");
+  asm volatile("fence.proxy.tensormap::generic.release.gpu;" ::: "memory");
 }
 
 }  // namespace tc

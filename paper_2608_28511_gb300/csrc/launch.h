@@ -112,6 +112,8 @@ struct GemmDesc {
   int64_t ldc = 0, sc_g = 0;
   const float* bias = nullptr;       // StoreBias
   void* aux = nullptr;               // SwigluFwd activation output (c_type)
+  void* scratch = nullptr;           // Group::K on the tensor-core engine: per-group tensor maps
+                                     // (gemm_tc_group_scratch_bytes, 128-byte aligned)
 };
 
 cudaError_t launch_gemm_simt(const Ctx& c, const GemmDesc& d, const char* name);
@@ -119,6 +121,7 @@ cudaError_t launch_gemm_simt(const Ctx& c, const GemmDesc& d, const char* name);
 // tcgen05 / TMA engine (bf16 operands only).  Returns cudaErrorNotSupported
 // for a descriptor it does not handle.
 bool gemm_tc_supports(const GemmDesc& d);
+size_t gemm_tc_group_scratch_bytes(int num_groups);
 cudaError_t launch_gemm_tc(const Ctx& c, const GemmDesc& d, const char* name);
 
 }  // namespace moe
