@@ -173,7 +173,24 @@ size_t ws_perm(const Dims& d) { return align_up(perm_workspace_bytes(d.TK, d.E))
 // dH [TK, 2F], dA [TK, F], then the wgrad GEMMs' per-expert tensor maps
 size_t ws_ffn_bwd_maps_offset(const Dims& d) { return align_up((size_t)d.TK * 3 * d.F * d.bx); }
 size_t ws_ffn_bwd(const Dims& d) { return ws_ffn_bwd_maps_offset(d) + align_up(gemm_tc_group_scratch_bytes(d.E)); }
-size_t ws_route_bwd(const Dims& d) { return align_up((size_t)d.T * d.E * 2); }
+// Router weight gradient: split-K over the T tokens into at most kRouterSplits
+// fp32 partial products, summed in order afterwards.
+constexpr int kRouterSplits = 16;
+size_t ws_route_dz(const Dims& d) { return align_up((size_t)d.T * d.E * 2); }
+size_t ws_route_parts(const Dims& d) { return align_up((size_t)kRouterSplits * d.E * d.Din * 4); }
+size_t ws_route_bwd(const Dims& d) {
+  return ws_route_dz(d) + ws_route_parts(d) + align_up(gemm_tc_group_scratch_bytes(kRouterSplits));
+}
+// Splits that fill the GPU: the output has ceil(E / tile rows) x ceil(Din / 256) tiles.
+int router_splits(const Dims& d, int num_sms) {
+  const bool pair = d.E > 128;
+  const int64_t tiles = ((d.E + (pair ? 255 : 127)) / (pair ? 256 : 128)) * ((d.Din + 255) / 256);
+  const int64_t slots = pair ? num_sms / 2 : num_sms;
+  int64_t s = slots / (tiles > 0 ? tiles : 1);
+  if (s > kRouterSplits) s = kRouterSplits;
+  if (s > d.T / 256) s = d.T / 256;
+  return s < 1 ? 1 : (int)s;
+}
 size_t ws_total(const Dims& d) {
   size_t m = ws_perm(d);
   m = std::max(m, ws_ffn_bwd(d));
@@ -649,6 +666,26 @@ int moe_route_bwd(const moe_shape_t* shape, const void* x, const void* w_router,
     if (gemm_tc_supports(b16)) b = b16;
   }
   if (d.T > 0) TRY_CUDA(gemm(c, a, "router_dgrad_tc", "router_dgrad_simt"));
+  const int splits = d.dt == DType::BF16 ? router_splits(d, c.num_sms) : 1;
+  if (splits > 1) {
+    // split-K: partial products of equal token ranges, then their in-order sum
+    GemmDesc bs = b;
+    bs.group = Group::K;
+    bs.num_groups = splits;
+    bs.offsets = nullptr;
+    bs.split_rows = d.T;
+    bs.max_rows = d.T;
+    bs.A = dz16;
+    bs.a_type = DType::BF16;
+    bs.C = static_cast<char*>(ws) + ws_route_dz(d);
+    bs.sc_g = (int64_t)d.E * d.Din;
+    bs.scratch = static_cast<char*>(ws) + ws_route_dz(d) + ws_route_parts(d);
+    if (gemm_tc_supports(bs)) {
+      TRY_CUDA(launch_gemm_tc(c, bs, "router_wgrad_tc"));
+      TRY_CUDA(launch_sum_splits(c, static_cast<const float*>(bs.C), splits, (int64_t)d.E * d.Din, dw_router));
+      return MOE_OK;
+    }
+  }
   TRY_CUDA(gemm(c, b, "router_wgrad_tc", "router_wgrad_simt"));
   return MOE_OK;
 }

@@ -69,9 +69,11 @@ bool make_plan(const GemmDesc& d, Plan* pl) {
   if (!al16(d.A) || !al16(d.B) || !al16(d.C)) return false;
   if (d.group == Group::K && !(pl->a_mn && pl->b_mn)) return false;
   if (d.group == Group::K && (!d.scratch || ((uintptr_t)d.scratch & 127u) || d.max_rows <= 0)) return false;
+  if (d.group == Group::K && !d.offsets && d.split_rows <= 0) return false;
   if (d.group == Group::M && pl->a_mn) return false;
   if (d.group == Group::M && (d.sb_g % pl->ldb)) return false;
-  if (d.group != Group::Dense && (d.num_groups <= 0 || d.num_groups > kMaxE || !d.offsets)) return false;
+  if (d.group != Group::Dense && (d.num_groups <= 0 || d.num_groups > kMaxE)) return false;
+  if (d.group == Group::M && !d.offsets) return false;
   const size_t cs = dsize(d.c_type);
   if ((d.ldc * cs) % 16) return false;
   switch (d.epi) {
@@ -156,7 +158,10 @@ cudaError_t launch_inst(const Ctx& c, const Params& p, int64_t ub) {
 
 }  // namespace
 
-size_t gemm_tc_group_scratch_bytes(int num_groups) { return (size_t)num_groups * 2 * sizeof(CUtensorMap); }
+// {A, B} map per group, then (for equal splits) the group offsets.
+size_t gemm_tc_group_scratch_bytes(int num_groups) {
+  return (size_t)num_groups * 2 * sizeof(CUtensorMap) + (((size_t)num_groups + 1) * 4 + 127) / 128 * 128;
+}
 
 bool gemm_tc_supports(const GemmDesc& d) {
   Plan pl;
@@ -215,15 +220,17 @@ cudaError_t launch_gemm_tc(const Ctx& c, const GemmDesc& d, const char* name) {
   if (d.group == Group::K) {
     // per-group maps: the templates above with the base and row extent moved per group
     CUtensorMap* maps = static_cast<CUtensorMap*>(d.scratch);
+    int32_t* split_offs = d.offsets ? nullptr : reinterpret_cast<int32_t*>(maps + 2 * d.num_groups);
     {
       KernelScope ks("group_maps", c.stream);
       tc::build_group_maps<<<(d.num_groups + 127) / 128, 128, 0, c.stream>>>(
-          p.ta, p.tb, d.offsets, d.num_groups, static_cast<const uint8_t*>(d.A), pl.lda * 2,
-          static_cast<const uint8_t*>(d.B), pl.ldb * 2, maps);
+          p.ta, p.tb, d.offsets, d.num_groups, d.split_rows, split_offs, static_cast<const uint8_t*>(d.A),
+          pl.lda * 2, static_cast<const uint8_t*>(d.B), pl.ldb * 2, maps);
     }
     cudaError_t st = cudaGetLastError();
     if (st != cudaSuccess) return st;
     p.gmaps = maps;
+    if (split_offs) p.offsets = split_offs;
   }
   KernelScope ks(name, c.stream);
   if (pl.cg == 2) {

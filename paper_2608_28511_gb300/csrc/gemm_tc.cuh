@@ -677,8 +677,16 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
         }
         continue;
       }
-      uint4 cur[4], nxt[4];  // an accumulating chunk's C block, fetched one chunk ahead
-      if (EPI == 2) acc_fetch(c_rows, ldc_b, n0, lane, nrows, cur);
+      // EPI 2: every chunk's C block is fetched before the accumulator wait, so
+      // the reads overlap the MMA and each other
+      constexpr int kPre = EPI == 2 ? BN / 32 : 1;
+      uint4 pre[kPre][4];
+      const int nch_acc = (int)imin64(BN / 32, (p.N - n0) / 32);
+      if (EPI == 2) {
+#pragma unroll
+        for (int c = 0; c < kPre; ++c)
+          if (c < nch_acc) acc_fetch(c_rows, ldc_b, n0 + c * 32, lane, nrows, pre[c]);
+      }
       if (!wait_bounded<CG == 2>(smem_u32(&tfull[acc]), acc_phase, &s_abort, p.err)) break;
       tc_fence_after();
       const uint32_t tbase = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
@@ -719,29 +727,27 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
           }
         }
       } else if (EPI == 2) {
-        // C += acc.  Chunk c + 1's C block is fetched into registers while
-        // chunk c is processed (chunk 0's before the accumulator wait).
-        const int nch = (int)imin64(BN / 32, (p.N - n0) / 32);
-        for (int c = 0; c < nch; ++c) {
-          const int64_t col0 = n0 + c * 32;
-          if (c + 1 < nch) acc_fetch(c_rows, ldc_b, col0 + 32, lane, nrows, nxt);
-          tmem_ld32(tbase + c * 32, v);
-          __syncwarp();
-          acc_put(stg, lane, cur);
-          __syncwarp();
-          stage_get<RB>(stg, lane, pk);
-          float o[32];
+        // C += acc, with the C blocks fetched above
 #pragma unroll
-          for (int i = 0; i < NP; ++i) unpack16<TC>(pk[i], o + i * Vec<TC>::N);
+        for (int c = 0; c < kPre; ++c) {
+          if (c < nch_acc) {
+            const int64_t col0 = n0 + c * 32;
+            tmem_ld32(tbase + c * 32, v);
+            __syncwarp();
+            acc_put(stg, lane, pre[c]);
+            __syncwarp();
+            stage_get<RB>(stg, lane, pk);
+            float o[32];
 #pragma unroll
-          for (int i = 0; i < 32; ++i) o[i] += v[i];
+            for (int i = 0; i < NP; ++i) unpack16<TC>(pk[i], o + i * Vec<TC>::N);
 #pragma unroll
-          for (int i = 0; i < NP; ++i) pk[i] = pack16<TC>(o + i * Vec<TC>::N);
-          stage_put<RB>(stg, lane, pk);
-          __syncwarp();
-          stage_store<RB>(stg, lane, c_rows + col0 * sizeof(TC), ldc_b, nrows);
+            for (int i = 0; i < 32; ++i) o[i] += v[i];
 #pragma unroll
-          for (int i = 0; i < 4; ++i) cur[i] = nxt[i];
+            for (int i = 0; i < NP; ++i) pk[i] = pack16<TC>(o + i * Vec<TC>::N);
+            stage_put<RB>(stg, lane, pk);
+            __syncwarp();
+            stage_store<RB>(stg, lane, c_rows + col0 * sizeof(TC), ldc_b, nrows);
+          }
         }
       } else {
 #pragma unroll 1
@@ -797,14 +803,25 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
 // the full-tensor templates with the base moved to the group's first row and
 // the row extent set to the group's row count (at least 1), so a copy that
 // runs past the group's rows reads zeros.  out[2g] = A, out[2g + 1] = B.
+// With offsets == nullptr the groups are G equal splits of [0, split_rows)
+// and their offsets are written to offs_out for the GEMM to read.
 __global__ void build_group_maps(const __grid_constant__ CUtensorMap ta, const __grid_constant__ CUtensorMap tb,
-                                 const int32_t* __restrict__ offsets, int G, const uint8_t* a_base,
-                                 int64_t a_row_bytes, const uint8_t* b_base, int64_t b_row_bytes,
-                                 CUtensorMap* out) {
+                                 const int32_t* __restrict__ offsets, int G, int64_t split_rows,
+                                 int32_t* __restrict__ offs_out, const uint8_t* a_base, int64_t a_row_bytes,
+                                 const uint8_t* b_base, int64_t b_row_bytes, CUtensorMap* out) {
   const int g = blockIdx.x * blockDim.x + threadIdx.x;
   if (g >= G) return;
-  const int64_t lo = offsets[g];
-  const int64_t rows = offsets[g + 1] - lo;
+  int64_t lo, hi;
+  if (offsets) {
+    lo = offsets[g];
+    hi = offsets[g + 1];
+  } else {
+    lo = split_rows * g / G;
+    hi = split_rows * (g + 1) / G;
+    offs_out[g] = (int32_t)lo;
+    if (g == G - 1) offs_out[G] = (int32_t)hi;
+  }
+  const int64_t rows = hi - lo;
   const uint32_t dim = rows > 0 ? (uint32_t)rows : 1u;
   CUtensorMap* ma = out + 2 * g;
   CUtensorMap* mb = ma + 1;

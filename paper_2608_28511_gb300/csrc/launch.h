@@ -51,6 +51,8 @@ constexpr int kMaxK = 16;
 constexpr int kMaxE = 256;
 
 cudaError_t launch_topk(const Ctx& c, const float* logits, int64_t T, int E, int K, int32_t* idx, float* prob);
+// out[i] = sum over s of part[s * n + i], s = 0 .. S-1 in order (fp32).
+cudaError_t launch_sum_splits(const Ctx& c, const float* part, int S, int64_t n, float* out);
 // dz[T, E] fp32 (fully written) and optionally a bf16 copy.
 cudaError_t launch_route_dz(const Ctx& c, const int32_t* idx, const float* prob, const float* dprob, int64_t T,
                             int E, int K, float* dz, void* dz_bf16);
@@ -114,6 +116,8 @@ struct GemmDesc {
   void* aux = nullptr;               // SwigluFwd activation output (c_type)
   void* scratch = nullptr;           // Group::K on the tensor-core engine: per-group tensor maps
                                      // (gemm_tc_group_scratch_bytes, 128-byte aligned)
+  int64_t split_rows = 0;            // Group::K with offsets == nullptr: num_groups equal splits of
+                                     // [0, split_rows) (split-K of a dense product)
 };
 
 cudaError_t launch_gemm_simt(const Ctx& c, const GemmDesc& d, const char* name);

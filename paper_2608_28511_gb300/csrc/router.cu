@@ -135,4 +135,30 @@ cudaError_t launch_route_dz(const Ctx& c, const int32_t* idx, const float* prob,
   return cudaGetLastError();
 }
 
+// Deterministic reduction of split-K partial products: each output is the
+// in-order sum of its S partials.
+__global__ void __launch_bounds__(256) sum_splits_kernel(const float4* __restrict__ part, int S, int64_t n4,
+                                                         float4* __restrict__ out) {
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n4; i += (int64_t)gridDim.x * blockDim.x) {
+    float4 a = __ldcs(part + i);
+    for (int s = 1; s < S; ++s) {
+      const float4 b = __ldcs(part + (int64_t)s * n4 + i);
+      a.x += b.x;
+      a.y += b.y;
+      a.z += b.z;
+      a.w += b.w;
+    }
+    out[i] = a;
+  }
+}
+
+cudaError_t launch_sum_splits(const Ctx& c, const float* part, int S, int64_t n, float* out) {
+  const int64_t n4 = n / 4;
+  const int64_t want = (n4 + 255) / 256;
+  const int blocks = (int)(want < (int64_t)c.num_sms * 8 ? want : (int64_t)c.num_sms * 8);
+  KernelScope ks("sum_splits", c.stream);
+  sum_splits_kernel<<<blocks, 256, 0, c.stream>>>((const float4*)part, S, n4, (float4*)out);
+  return cudaGetLastError();
+}
+
 }  // namespace moe
