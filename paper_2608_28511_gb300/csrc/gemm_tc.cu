@@ -96,10 +96,10 @@ bool make_plan(const GemmDesc& d, Plan* pl) {
 
 // Co-resident 2-CTA clusters of an instantiation (0 if the query fails).
 template <typename KernelT>
-int max_pair_clusters(KernelT k, int smem) {
+int max_pair_clusters(KernelT k, int smem, int threads) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(2, 1, 1);
-  cfg.blockDim = dim3(tc::kThreads, 1, 1);
+  cfg.blockDim = dim3(threads, 1, 1);
   cfg.dynamicSmemBytes = smem;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -120,7 +120,8 @@ int max_pair_clusters(KernelT k, int smem) {
 template <int BN, bool A_MN, bool B_MN, int GROUP, int EPI, typename TC, int CG>
 cudaError_t launch_inst(const Ctx& c, const Params& p, int64_t ub) {
   auto k = tc::gemm_tc_kernel<BN, A_MN, B_MN, GROUP, EPI, TC, CG>;
-  constexpr int kSmem = Cfg<BN, CG>::kSmem;
+  constexpr int kSmem = Cfg<BN, CG, sizeof(TC)>::kSmem;
+  constexpr int kThreads = Cfg<BN, CG, sizeof(TC)>::kThreads;
   static bool configured = false;
   static int pairs = 0;
   if (!configured) {
@@ -130,20 +131,20 @@ cudaError_t launch_inst(const Ctx& c, const Params& p, int64_t ub) {
       e = cudaFuncSetAttribute(k, cudaFuncAttributeNonPortableClusterSizeAllowed, 0);
       (void)e;
       cudaGetLastError();
-      pairs = max_pair_clusters(k, kSmem);
+      pairs = max_pair_clusters(k, kSmem, kThreads);
     }
     configured = true;
   }
   if (CG == 1) {
     const int grid = (int)(ub < c.num_sms ? ub : c.num_sms);
-    k<<<grid, tc::kThreads, kSmem, c.stream>>>(p);
+    k<<<grid, kThreads, kSmem, c.stream>>>(p);
     return cudaGetLastError();
   }
   int np = pairs > 0 ? pairs : c.num_sms / 2;
   if (ub < np) np = (int)ub;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(2 * np, 1, 1);
-  cfg.blockDim = dim3(tc::kThreads, 1, 1);
+  cfg.blockDim = dim3(kThreads, 1, 1);
   cfg.dynamicSmemBytes = kSmem;
   cfg.stream = c.stream;
   cudaLaunchAttribute attr[1];

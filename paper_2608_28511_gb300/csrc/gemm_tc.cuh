@@ -3,11 +3,12 @@
 //
 // C(m, n) = sum_k A(m, k) B(n, k) over 128 x BN x 64 tiles.  One persistent
 // CTA per SM walks a static tile sequence decoded on the device from the
-// expert offsets (no host synchronisation).  Warp roles (192 threads):
+// expert offsets (no host synchronisation).  Warp roles:
 //   warp 0      TMA producer (one lane) filling a kStages-deep smem ring;
 //   warp 1      TMEM allocator and MMA issuer (one lane issues, all wait);
-//   warps 2..5  epilogue: TMEM -> registers -> global, one accumulator row
-//               per thread, double-buffered accumulators (2 x BN columns).
+//   warps 2..   epilogue (4, or 8 for bf16 outputs): TMEM -> registers ->
+//               global, one accumulator row per thread, double-buffered
+//               accumulators (2 x BN columns).
 // Operands are staged with 128-byte swizzle; A and B may each be K-major
 // (rows of K contiguous) or MN-major (rows of M / N contiguous).
 //
@@ -30,7 +31,6 @@ namespace tc {
 
 constexpr int BM = 128;
 constexpr int BK = 64;                  // bf16: 128 bytes, one swizzle row
-constexpr int kThreads = 192;
 constexpr uint64_t kWaitLimitNs = 4000000000ull;
 
 struct Params {
@@ -291,7 +291,7 @@ __host__ __device__ constexpr uint32_t make_idesc(int bn, int bm, bool a_mn, boo
 // CG = 1: one CTA computes a 128 x BN tile.  CG = 2: a cluster of two CTAs
 // computes a 256 x BN tile; each CTA stages its 128 rows of A and BN / 2 rows
 // of B, and holds its 128 accumulator rows in its own TMEM.
-template <int BN, int CG = 1>
+template <int BN, int CG = 1, int TCB = 2>  // TCB: bytes per element of C
 struct Cfg {
   static constexpr int kBRows = BN / CG;
   static constexpr int kABytes = BM * BK * 2;
@@ -299,16 +299,23 @@ struct Cfg {
   static constexpr int kStageBytes = kABytes + kBBytes;
   static constexpr int kStages = (196608 / kStageBytes) < 8 ? (196608 / kStageBytes) : 8;
   static constexpr int kCols = 2 * BN;  // double-buffered fp32 accumulator
-  // per epilogue warp: 32 rows x 128 B staging, rows padded to 144 B (conflict-free both ways)
-  static constexpr int kPitch = 144;
+  // Epilogue warps: 8 (two per TMEM lane quarter, each taking half the
+  // columns) for bf16 outputs, whose epilogues are latency-bound; 4 for fp32
+  // outputs, which are bound by their store bandwidth.
+  static constexpr int kEpiWarps = TCB == 2 ? 8 : 4;
+  static constexpr int kThreads = 64 + 32 * kEpiWarps;
+  // per epilogue warp: 32 rows x 32 columns of C staging, rows padded by 16 B
+  // (conflict-free both ways)
+  static constexpr int kRowBytes = 32 * TCB;
+  static constexpr int kPitch = kRowBytes + 16;
   static constexpr int kStageBufBytes = 32 * kPitch;
-  static constexpr int kStagingBytes = 4 * kStageBufBytes;
+  static constexpr int kStagingBytes = kEpiWarps * kStageBufBytes;
   static constexpr int kSmem = kStages * kStageBytes + kStagingBytes + 1024 /*align*/ + 512 /*barriers*/;
 };
 
 // ---------------------------------------------------------------------------
 // Epilogue staging: each epilogue warp owns 32 accumulator rows (one per
-// lane).  A lane writes its row into the warp's staging buffer, then the warp
+// lane) of its share of the columns.  A lane writes its row into the warp's staging buffer, then the warp
 // copies the 32 rows to global memory with lanes covering consecutive 16-byte
 // pieces of a row, so every store instruction writes whole 128-byte lines
 // instead of 32 scattered half-sectors.  Loads of epilogue inputs (the saved
@@ -317,12 +324,12 @@ struct Cfg {
 template <int NB>  // bytes per row: 64 or 128
 __device__ __forceinline__ void stage_put(uint8_t* buf, int lane, const uint4* row) {
 #pragma unroll
-  for (int j = 0; j < NB / 16; ++j) *reinterpret_cast<uint4*>(buf + lane * 144 + j * 16) = row[j];
+  for (int j = 0; j < NB / 16; ++j) *reinterpret_cast<uint4*>(buf + lane * (NB + 16) + j * 16) = row[j];
 }
 template <int NB>
 __device__ __forceinline__ void stage_get(const uint8_t* buf, int lane, uint4* row) {
 #pragma unroll
-  for (int j = 0; j < NB / 16; ++j) row[j] = *reinterpret_cast<const uint4*>(buf + lane * 144 + j * 16);
+  for (int j = 0; j < NB / 16; ++j) row[j] = *reinterpret_cast<const uint4*>(buf + lane * (NB + 16) + j * 16);
 }
 // buf rows 0..31 -> gbase + r * ld_bytes (rows r >= nrows are skipped).
 template <int NB>
@@ -332,13 +339,13 @@ __device__ __forceinline__ void stage_store(const uint8_t* buf, int lane, uint8_
 #pragma unroll
   for (int it = 0; it < 32 / RPI; ++it) {
     const int r = it * RPI + lane / CPR, c = lane % CPR;
-    const uint4 v = *reinterpret_cast<const uint4*>(buf + r * 144 + c * 16);
+    const uint4 v = *reinterpret_cast<const uint4*>(buf + r * (NB + 16) + c * 16);
     if (r < nrows) *reinterpret_cast<uint4*>(gbase + r * ld_bytes + c * 16) = v;
   }
 }
 // The 32 x 32 bf16 block of C an accumulating chunk adds to, fetched into
 // registers as 16-byte pieces (4 per lane; rows >= nrows as zero), and put
-// into the staging buffer in row order.
+// into the staging buffer in row order (64-byte rows, 80-byte pitch).
 __device__ __forceinline__ void acc_fetch(const uint8_t* rows, int64_t ld_b, int64_t col0, int lane, int nrows,
                                           uint4* dst) {
 #pragma unroll
@@ -352,7 +359,7 @@ __device__ __forceinline__ void acc_put(uint8_t* buf, int lane, const uint4* src
 #pragma unroll
   for (int it = 0; it < 4; ++it) {
     const int r = it * 8 + lane / 4, pc = lane % 4;
-    *reinterpret_cast<uint4*>(buf + r * 144 + pc * 16) = src[it];
+    *reinterpret_cast<uint4*>(buf + r * 80 + pc * 16) = src[it];
   }
 }
 // gbase + r * ld_bytes -> buf rows 0..31 (rows r >= nrows read as zero).
@@ -365,7 +372,7 @@ __device__ __forceinline__ void stage_load(uint8_t* buf, int lane, const uint8_t
     const int r = it * RPI + lane / CPR, c = lane % CPR;
     uint4 v = make_uint4(0, 0, 0, 0);
     if (r < nrows) v = *reinterpret_cast<const uint4*>(gbase + r * ld_bytes + c * 16);
-    *reinterpret_cast<uint4*>(buf + r * 144 + c * 16) = v;
+    *reinterpret_cast<uint4*>(buf + r * (NB + 16) + c * 16) = v;
   }
 }
 
@@ -419,8 +426,15 @@ __device__ __forceinline__ void decode_tile(const Params& p, int t, const int* s
 __device__ __forceinline__ int64_t imin64(int64_t a, int64_t b) { return a < b ? a : b; }
 __device__ __forceinline__ int64_t imax64(int64_t a, int64_t b) { return a > b ? a : b; }
 
-__device__ __forceinline__ float silu_f(float v) { return v / (1.0f + __expf(-v)); }
-__device__ __forceinline__ float sigmoid_f(float v) { return 1.0f / (1.0f + __expf(-v)); }
+// silu(v) = v sigmoid(v) with sigmoid(v) = (1 + tanh(v / 2)) / 2 on the
+// hardware tanh approximation (one MUFU op; its ~5e-4 error is far below
+// the bf16 rounding of the stored activation).
+__device__ __forceinline__ float tanh_approx(float x) {
+  float y;
+  asm("tanh.approx.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+__device__ __forceinline__ float silu_f(float v) { return v * fmaf(0.5f, tanh_approx(0.5f * v), 0.5f); }
 
 template <typename T>
 __device__ __forceinline__ void store_row32(T* dst, const float* v, int valid) {
@@ -446,8 +460,11 @@ __device__ __forceinline__ void load_row32(const T* src, float* v) {
 // tile (the even CTA issues the MMAs; both stage their halves and drain
 // their own accumulator rows).
 template <int BN, bool A_MN, bool B_MN, int GROUP, int EPI, typename TC, int CG>
-__global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_constant__ Params p) {
-  using C = Cfg<BN, CG>;
+__global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
+    gemm_tc_kernel(const __grid_constant__ Params p) {
+  using C = Cfg<BN, CG, sizeof(TC)>;
+  constexpr int EW = C::kEpiWarps;
+  constexpr int CSTEP = EW / 4;  // epilogue warps sharing a lane quarter
   constexpr int BMP = BM * CG;
   constexpr int BNC = C::kBRows;
   constexpr uint32_t kIdesc = make_idesc(BN, BMP, A_MN, B_MN);
@@ -478,7 +495,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(smem_u32(&tfull[a]), 1);
-      mbar_init(smem_u32(&tempty[a]), 4 * CG);
+      mbar_init(smem_u32(&tempty[a]), EW * CG);
     }
     mbar_init(smem_u32(done), 1);
     fence_barrier_init();
@@ -491,7 +508,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     tmem_relinquish_cg<CG>();
   }
   if (GROUP != 0) {
-    for (int i = tid; i <= p.num_groups; i += kThreads) s_off[i] = p.offsets[i];
+    for (int i = tid; i <= p.num_groups; i += C::kThreads) s_off[i] = p.offsets[i];
   }
   __syncthreads();
   if (tid == 0) {
@@ -638,10 +655,14 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     __syncwarp();
   } else {
     // ------------------------------------------------------------ epilogue
-    const int q = warp & 3;
-    uint8_t* stg = smem + C::kStages * C::kStageBytes + q * C::kStageBufBytes;
-    constexpr int RB = (int)sizeof(TC) * 32;  // bytes of 32 columns of C
-    constexpr int NP = RB / 16;               // 16-byte pieces per 32 columns
+    const int q = warp & 3;            // TMEM lane quarter
+    const int ew = warp - 2;
+    const int ch = ew >> 2;            // which of the CSTEP column interleaves this warp takes
+    uint8_t* stg = smem + C::kStages * C::kStageBytes + ew * C::kStageBufBytes;
+    constexpr int RB = C::kRowBytes;               // bytes per staged row (32 columns)
+    constexpr int NP = RB / 16;                    // 16-byte pieces per staged row
+    constexpr int RPC = (int)sizeof(TC) * 32 / RB; // rounds per 32-column chunk (1)
+    constexpr int CPR = RB / (int)sizeof(TC);      // columns per round
     const int64_t ldc_b = p.ldc * (int64_t)sizeof(TC);
     int acc = 0;
     uint32_t acc_phase = 0;
@@ -660,14 +681,17 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
         uint4 z[NP];
 #pragma unroll
         for (int i = 0; i < NP; ++i) z[i] = make_uint4(0, 0, 0, 0);
-        for (int c = 0; c < BN / 32; ++c) {
+        for (int c = ch; c < BN / 32; c += CSTEP) {
           const int64_t col0 = n0 + c * 32;
           if (col0 >= p.N) break;
           if (p.N - col0 >= 32) {
-            __syncwarp();
-            stage_put<RB>(stg, lane, z);
-            __syncwarp();
-            stage_store<RB>(stg, lane, c_rows + col0 * sizeof(TC), ldc_b, nrows);
+#pragma unroll
+            for (int r = 0; r < RPC; ++r) {
+              __syncwarp();
+              stage_put<RB>(stg, lane, z);
+              __syncwarp();
+              stage_store<RB>(stg, lane, c_rows + (col0 + r * CPR) * sizeof(TC), ldc_b, nrows);
+            }
           } else if (vrow) {
             float zf[32];
 #pragma unroll
@@ -679,13 +703,13 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
       }
       // EPI 2: every chunk's C block is fetched before the accumulator wait, so
       // the reads overlap the MMA and each other
-      constexpr int kPre = EPI == 2 ? BN / 32 : 1;
+      constexpr int kPre = EPI == 2 ? BN / 32 / CSTEP : 1;  // this warp's chunks: ch, ch + CSTEP, ...
       uint4 pre[kPre][4];
       const int nch_acc = (int)imin64(BN / 32, (p.N - n0) / 32);
       if (EPI == 2) {
 #pragma unroll
-        for (int c = 0; c < kPre; ++c)
-          if (c < nch_acc) acc_fetch(c_rows, ldc_b, n0 + c * 32, lane, nrows, pre[c]);
+        for (int i = 0; i < kPre; ++i)
+          if (ch + i * CSTEP < nch_acc) acc_fetch(c_rows, ldc_b, n0 + (ch + i * CSTEP) * 32, lane, nrows, pre[i]);
       }
       if (!wait_bounded<CG == 2>(smem_u32(&tfull[acc]), acc_phase, &s_abort, p.err)) break;
       tc_fence_after();
@@ -696,11 +720,12 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
         // packed [gate 64 | up 64] blocks: h = [g | u] stored as computed, a = silu(g) * u
         uint8_t* a_rows = reinterpret_cast<uint8_t*>(static_cast<TC*>(p.aux) + rbase * (p.N / 2));
         const int64_t lda_b = (p.N / 2) * (int64_t)sizeof(TC);
-        for (int blk = 0; blk < BN / 128; ++blk) {
+#pragma unroll 1
+        for (int hb = ch; hb < BN / 64; hb += CSTEP) {  // half-blocks: 32 gate + 32 up columns
+          const int blk = hb >> 1, half = hb & 1;
           const int64_t cb = n0 + blk * 128;
           if (cb >= p.N) break;
-#pragma unroll 1
-          for (int half = 0; half < 2; ++half) {
+          {
             float u[32], a[32];
             tmem_ld32(tbase + blk * 128 + half * 32, v);
             tmem_ld32(tbase + blk * 128 + 64 + half * 32, u);
@@ -729,12 +754,13 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
       } else if (EPI == 2) {
         // C += acc, with the C blocks fetched above
 #pragma unroll
-        for (int c = 0; c < kPre; ++c) {
+        for (int i = 0; i < kPre; ++i) {
+          const int c = ch + i * CSTEP;
           if (c < nch_acc) {
             const int64_t col0 = n0 + c * 32;
             tmem_ld32(tbase + c * 32, v);
             __syncwarp();
-            acc_put(stg, lane, pre[c]);
+            acc_put(stg, lane, pre[i]);
             __syncwarp();
             stage_get<RB>(stg, lane, pk);
             float o[32];
@@ -751,7 +777,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
         }
       } else {
 #pragma unroll 1
-        for (int c = 0; c < BN / 32; ++c) {
+        for (int c = ch; c < BN / 32; c += CSTEP) {
           const int64_t col0 = n0 + c * 32;
           if (col0 >= p.N) break;
           tmem_ld32(tbase + c * 32, v);
@@ -773,11 +799,14 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
             store_row32<TC>(crow + col0, v, nvalid);
           } else if (EPI == 0) {
 #pragma unroll
-            for (int i = 0; i < NP; ++i) pk[i] = pack16<TC>(v + i * Vec<TC>::N);
-            __syncwarp();
-            stage_put<RB>(stg, lane, pk);
-            __syncwarp();
-            stage_store<RB>(stg, lane, c_rows + col0 * sizeof(TC), ldc_b, nrows);
+            for (int r = 0; r < RPC; ++r) {
+#pragma unroll
+              for (int i = 0; i < NP; ++i) pk[i] = pack16<TC>(v + r * CPR + i * Vec<TC>::N);
+              __syncwarp();
+              stage_put<RB>(stg, lane, pk);
+              __syncwarp();
+              stage_store<RB>(stg, lane, c_rows + (col0 + r * CPR) * sizeof(TC), ldc_b, nrows);
+            }
           }
         }
       }
