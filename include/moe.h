@@ -206,6 +206,28 @@ int moe_pack_w1(const moe_shape_t* shape, const void* w_gate, const void* w_up, 
  * S * GBS * K * (4 D b_x + 2 b_p), b_p = 4.  Host only; 0 on a bad shape. */
 uint64_t moe_eq1_bytes(const moe_shape_t* shape);
 
+/* ---- CE-MoE layout tools (host only) ------------------------------------
+ * Layer composition (Sec. 4.1): from a baseline of a_star Mamba, b_star MoE
+ * and c_star attention blocks (L = a_star + b_star + c_star) and a target
+ * token-mixing-to-MoE ratio alpha, the CE-MoE composition keeps c = c_star,
+ * sets b = d = floor(L / (alpha + 2)) MoE and dense-FFN blocks and gives the
+ * rest to Mamba: a = L - b - c - d.  MOE_ERR_SHAPE if a would be negative. */
+int moe_ce_composition(int32_t a_star, int32_t b_star, int32_t c_star, double alpha, int32_t* a, int32_t* b,
+                       int32_t* c, int32_t* d);
+
+/* Layer pattern of Algorithm 1 (Sec. 4.2) for a composition (a Mamba, b MoE,
+ * c attention, d dense FFN; b >= c).  Writes the pattern over M, E, * and -
+ * into `pattern` (NUL-terminated), the virtual-block order over A / N / R into
+ * `blocks` and the pattern with A blocks in [ ] and N / R blocks in ( ) into
+ * `decorated` (either may be NULL).  Readings where the algorithm is loose:
+ * Distribute gives the N blocks near-equal groups of A blocks between them,
+ * larger groups first; Phase 3 makes one residue block per remaining MoE,
+ * attention or dense block (at least one) and shares the remaining Mamba
+ * evenly, larger shares first.  Returns the pattern length, or MOE_ERR_SHAPE
+ * (bad counts, or a buffer too small) / MOE_ERR_NULL. */
+int moe_ce_layer_pattern(int32_t a, int32_t b, int32_t c, int32_t d, char* pattern, size_t pattern_cap,
+                         char* blocks, size_t blocks_cap, char* decorated, size_t decorated_cap);
+
 /* Synchronises `stream`, then returns MOE_OK, MOE_ERR_DEVICE if the device
  * status word of the current device is set (and clears it), or MOE_ERR_CUDA.
  * Off the timed path. */

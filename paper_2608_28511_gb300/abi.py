@@ -32,6 +32,7 @@ EXPORTS = (
     "moe_latent_proj_bwd", "moe_pack_w1", "moe_eq1_bytes", "moe_check_device_status",
     "moe_device_status_word", "moe_last_cuda_error", "moe_strerror", "moe_version", "moe_prof_enable",
     "moe_prof_reset", "moe_prof_count", "moe_prof_get", "moe_launch_count", "moe_dispatch_noalloc",
+    "moe_ce_composition", "moe_ce_layer_pattern",
 )
 
 
@@ -97,6 +98,9 @@ _SIGS = {
                       ctypes.POINTER(ctypes.c_double)], ctypes.c_int),
     "moe_launch_count": ([], ctypes.c_uint64),
     "moe_dispatch_noalloc": ([_SHP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP], ctypes.c_int),
+    "moe_ce_composition": ([_I32, _I32, _I32, ctypes.c_double] + [ctypes.POINTER(_I32)] * 4, ctypes.c_int),
+    "moe_ce_layer_pattern": ([_I32, _I32, _I32, _I32, ctypes.c_char_p, _SZ, ctypes.c_char_p, _SZ, ctypes.c_char_p,
+                              _SZ], ctypes.c_int),
 }
 
 
@@ -283,3 +287,25 @@ def moe_prof_read() -> dict:
         _check("moe_prof_get", L.moe_prof_get(i, ctypes.byref(name), ctypes.byref(n), ctypes.byref(ms)))
         out[name.value.decode()] = (n.value, ms.value)
     return out
+
+
+# ---------------------------------------------------------------------------
+# CE-MoE layout tools (host only)
+# ---------------------------------------------------------------------------
+
+def moe_ce_composition(a_star: int, b_star: int, c_star: int, alpha: float) -> tuple:
+    """(a, b, c, d): Mamba, MoE, attention and dense-FFN block counts (Sec. 4.1)."""
+    out = [ctypes.c_int32(0) for _ in range(4)]
+    _check("moe_ce_composition", lib().moe_ce_composition(int(a_star), int(b_star), int(c_star), float(alpha),
+                                                          *[ctypes.byref(o) for o in out]))
+    return tuple(o.value for o in out)
+
+
+def moe_ce_layer_pattern(a: int, b: int, c: int, d: int) -> tuple:
+    """(pattern, virtual-block order, decorated pattern) of Algorithm 1 (Sec. 4.2)."""
+    cap = 4 * (a + b + c + d) + 64
+    bufs = [ctypes.create_string_buffer(cap) for _ in range(3)]
+    n = lib().moe_ce_layer_pattern(int(a), int(b), int(c), int(d), bufs[0], cap, bufs[1], cap, bufs[2], cap)
+    if n < 0:
+        _check("moe_ce_layer_pattern", n)
+    return tuple(b_.value.decode() for b_ in bufs)
