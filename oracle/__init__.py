@@ -7,3 +7,4 @@ or executes anything here, and this package imports nothing from the product.
 """
 from .moe import *  # noqa: F401,F403
 from .eq1 import *  # noqa: F401,F403
+from .router_sigmoid import *  # noqa: F401,F403

@@ -121,3 +121,27 @@ def test_wrong_combine_weight_is_caught(monkeypatch):
         return y
     _patch(monkeypatch, "combine", bad)
     _expect_failure(P.test_combine_of_dispatch_with_identity_experts_returns_x)
+
+
+def test_sigmoid_router_mistakes_are_caught(monkeypatch):
+    import oracle.router_sigmoid as RS
+    import tests.test_oracle_sigmoid as PS
+    orig_bwd = RS.sigmoid_route_bwd
+
+    def no_sigmoid_slope(x, w_router, z, idx, prob, dprob, f, S, GBS, coef, aux_grad=1.0):
+        dz, _, _ = orig_bwd(x, w_router, z, idx, prob, dprob, f, S, GBS, coef, aux_grad)
+        s = M.sigmoid(z)
+        dz = dz / (s * (1 - s))                       # dropped the sigmoid derivative
+        return dz, dz @ w_router, dz.T @ x
+    monkeypatch.setattr(RS, "sigmoid_route_bwd", no_sigmoid_slope)
+    monkeypatch.setattr(oracle, "sigmoid_route_bwd", no_sigmoid_slope)
+    _expect_failure(PS.test_router_gradient_matches_central_differences)
+
+    orig_aux = RS.seq_aux_loss
+
+    def wrong_fraction(z, idx, S, GBS, coef):
+        loss, f, P = orig_aux(z, idx, S, GBS, coef)
+        return loss * idx.shape[1], f * idx.shape[1], P     # missing the 1/K of the load fraction
+    monkeypatch.setattr(RS, "seq_aux_loss", wrong_fraction)
+    monkeypatch.setattr(oracle, "seq_aux_loss", wrong_fraction)
+    _expect_failure(PS.test_balanced_routing_with_flat_scores_gives_the_coefficient)
