@@ -186,6 +186,38 @@ int moe_route_bwd(const moe_shape_t* shape, const void* x, const void* w_router,
                   const float* topk_prob, const float* dtopk_prob, void* dx, float* dw_router, float* dlogits,
                   void* ws, size_t ws_bytes, void* stream);
 
+/* Sigmoid router with expert bias and the sequence-level balance loss
+ * (Sec. 5.2 experimental details; the paper gives no formulas, readings S1-S3):
+ *   logits[T, E] = x[T, Din] . w_router^T (fp32, no logit bias);
+ *   s = sigmoid(logits); the K experts with the largest s + expert_bias
+ *   (ties to the lower expert index, slots by descending s + b) -> topk_idx;
+ *   topk_prob[t, k] = s_k / sum over the K chosen of s (the bias shapes the
+ *   choice only);
+ *   sequence g = tokens g*S .. g*S+S-1 (shape->S tokens, shape->GBS sequences):
+ *   aux_f[g, i] = E / (K S) * #{t in g : i chosen}  ([GBS, E] fp32, written),
+ *   P[g, i] = mean over t in g of s_ti / sum_j s_tj,
+ *   aux_loss[0] = aux_coef / GBS * sum_{g,i} aux_f[g, i] P[g, i]  (fp32).
+ * expert_bias [E] fp32 may be NULL (zero).  Every reduction runs in a fixed
+ * order: results are bit-reproducible.  A NaN aux_coef is MOE_ERR_SHAPE. */
+int moe_route_sigmoid(const moe_shape_t* shape, const void* x, const void* w_router, const float* expert_bias,
+                      float aux_coef, float* logits, int32_t* topk_idx, float* topk_prob, float* aux_f,
+                      float* aux_loss, void* ws, size_t ws_bytes, void* stream);
+
+/* Sigmoid router backward: gradient of (the downstream loss through
+ * topk_prob, given as dtopk_prob [T, K]) + aux_grad * aux_loss with respect to
+ * the logits, with aux_f from moe_route_sigmoid (a count: no gradient) and
+ * c_gi = aux_grad * aux_coef / (GBS S) * aux_f[g, i]:
+ *   dL/ds_j = [j chosen] (dp_j - sum_k p_k dp_k) / sum_{chosen} s
+ *             + (c_gj - sum_i c_gi s_i / sum s) / sum_i s_i,
+ *   dlogits[t, j] = s_j (1 - s_j) dL/ds_j  ([T, E] fp32, fully written);
+ * then dx[T, Din] += dlogits . w_router (one rounding) and
+ * dw_router [E, Din] = dlogits^T . x (fp32, overwritten), as moe_route_bwd.
+ * The expert bias gets no gradient.  logits are moe_route_sigmoid's. */
+int moe_route_sigmoid_bwd(const moe_shape_t* shape, const void* x, const void* w_router, const float* logits,
+                          const int32_t* topk_idx, const float* topk_prob, const float* dtopk_prob,
+                          const float* aux_f, float aux_coef, float aux_grad, void* dx, float* dw_router,
+                          float* dlogits, void* ws, size_t ws_bytes, void* stream);
+
 /* LatentMoE projection (dense, T rows): out[T, n_out] = in[T, n_in] . w^T with
  * w [n_out, n_in].  Down-projection: n_in = H, n_out = D; up-projection:
  * n_in = D, n_out = H. */

@@ -27,16 +27,23 @@ from .moe import sigmoid
 __all__ = ["sigmoid_route", "seq_aux_loss", "sigmoid_route_bwd"]
 
 
-def sigmoid_route(z: np.ndarray, K: int, expert_bias=None):
-    """Readings S1, S2.  Returns idx [T, K] int64 and prob [T, K] float64."""
+def sigmoid_route(z: np.ndarray, K: int, expert_bias=None, idx_override=None):
+    """Readings S1, S2.  Returns idx [T, K] int64 and prob [T, K] float64.
+
+    ``idx_override`` replaces the choice (where a near-tie of s + b could
+    resolve either way); the gate values are then S2 over the given set.
+    """
     T, E = z.shape
     s = sigmoid(z)
     b = np.zeros(E) if expert_bias is None else np.asarray(expert_bias, dtype=np.float64)
     idx = np.empty((T, K), dtype=np.int64)
     prob = np.empty((T, K))
     for t in range(T):
-        key = [s[t, e] + b[e] for e in range(E)]
-        chosen = sorted(range(E), key=lambda e: (-key[e], e))[:K]
+        if idx_override is not None:
+            chosen = [int(e) for e in idx_override[t]]
+        else:
+            key = [s[t, e] + b[e] for e in range(E)]
+            chosen = sorted(range(E), key=lambda e: (-key[e], e))[:K]
         denom = sum(s[t, e] for e in chosen)
         for k, e in enumerate(chosen):
             idx[t, k] = e

@@ -32,7 +32,7 @@ EXPORTS = (
     "moe_latent_proj_bwd", "moe_pack_w1", "moe_eq1_bytes", "moe_check_device_status",
     "moe_device_status_word", "moe_last_cuda_error", "moe_strerror", "moe_version", "moe_prof_enable",
     "moe_prof_reset", "moe_prof_count", "moe_prof_get", "moe_launch_count", "moe_dispatch_noalloc",
-    "moe_ce_composition", "moe_ce_layer_pattern",
+    "moe_ce_composition", "moe_ce_layer_pattern", "moe_route_sigmoid", "moe_route_sigmoid_bwd",
 )
 
 
@@ -69,6 +69,7 @@ _lib = None
 _VP = ctypes.c_void_p
 _SZ = ctypes.c_size_t
 _I32 = ctypes.c_int32
+_F32 = ctypes.c_float
 _SHP = ctypes.POINTER(MoeShape)
 
 _SIGS = {
@@ -82,6 +83,9 @@ _SIGS = {
     "moe_expert_ffn_bwd": ([_SHP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _SZ, _VP], ctypes.c_int),
     "moe_dispatch_bwd": ([_SHP, _VP, _VP, _VP, _VP, _VP, _VP], ctypes.c_int),
     "moe_route_bwd": ([_SHP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _SZ, _VP], ctypes.c_int),
+    "moe_route_sigmoid": ([_SHP, _VP, _VP, _VP, _F32, _VP, _VP, _VP, _VP, _VP, _VP, _SZ, _VP], ctypes.c_int),
+    "moe_route_sigmoid_bwd": ([_SHP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _F32, _F32, _VP, _VP, _VP, _VP, _SZ, _VP],
+                              ctypes.c_int),
     "moe_latent_proj": ([_SHP, _I32, _I32, _VP, _VP, _VP, _VP, _SZ, _VP], ctypes.c_int),
     "moe_latent_proj_bwd": ([_SHP, _I32, _I32, _VP, _VP, _VP, _VP, _I32, _VP, _VP, _SZ, _VP], ctypes.c_int),
     "moe_pack_w1": ([_SHP, _VP, _VP, _VP, _VP], ctypes.c_int),
@@ -225,6 +229,21 @@ def moe_route_bwd(shape, x, w_router, topk_idx, topk_prob, dtopk_prob, dx, dw_ro
     _check("moe_route_bwd", lib().moe_route_bwd(_shape(shape), _p(x), _p(w_router), _p(topk_idx), _p(topk_prob),
                                                 _p(dtopk_prob), _p(dx), _p(dw_router), _p(dlogits), _p(ws),
                                                 _nbytes(ws), _stream(stream)))
+
+
+def moe_route_sigmoid(shape, x, w_router, expert_bias, aux_coef, logits, topk_idx, topk_prob, aux_f, aux_loss, ws,
+                      stream=None):
+    _check("moe_route_sigmoid", lib().moe_route_sigmoid(
+        _shape(shape), _p(x), _p(w_router), _p(expert_bias), float(aux_coef), _p(logits), _p(topk_idx),
+        _p(topk_prob), _p(aux_f), _p(aux_loss), _p(ws), _nbytes(ws), _stream(stream)))
+
+
+def moe_route_sigmoid_bwd(shape, x, w_router, logits, topk_idx, topk_prob, dtopk_prob, aux_f, aux_coef, aux_grad,
+                          dx, dw_router, dlogits, ws, stream=None):
+    _check("moe_route_sigmoid_bwd", lib().moe_route_sigmoid_bwd(
+        _shape(shape), _p(x), _p(w_router), _p(logits), _p(topk_idx), _p(topk_prob), _p(dtopk_prob), _p(aux_f),
+        float(aux_coef), float(aux_grad), _p(dx), _p(dw_router), _p(dlogits), _p(ws), _nbytes(ws),
+        _stream(stream)))
 
 
 def moe_latent_proj(shape, n_in, n_out, x, w, out, ws, stream=None):

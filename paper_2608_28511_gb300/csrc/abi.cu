@@ -117,7 +117,7 @@ int cuda_status(cudaError_t e) {
 
 // ---- validation -----------------------------------------------------------
 struct Dims {
-  int64_t T, TK;
+  int64_t S, GBS, T, TK;
   int K, D, E, F, H, Din;
   DType dt;
   size_t bx;
@@ -134,6 +134,8 @@ int check_shape(const moe_shape_t* s, Dims* d) {
   const int64_t T = s->S * s->GBS;
   const int64_t TK = T * s->K;
   if (TK >= (int64_t(1) << 31)) return MOE_ERR_SHAPE;
+  d->S = s->S;
+  d->GBS = s->GBS;
   d->T = T;
   d->TK = TK;
   d->K = s->K;
@@ -191,8 +193,12 @@ int router_splits(const Dims& d, int num_sms) {
   if (s > d.T / 256) s = d.T / 256;
   return s < 1 ? 1 : (int)s;
 }
+// Sigmoid router forward: per-token score sums and the balance statistics'
+// per-chunk partial sums.
+size_t ws_route_sigmoid(const Dims& d) { return align_up(route_sigmoid_fwd_ws_bytes(d.T, d.S, d.GBS, d.E)); }
 size_t ws_total(const Dims& d) {
   size_t m = ws_perm(d);
+  m = std::max(m, ws_route_sigmoid(d));
   m = std::max(m, ws_ffn_bwd(d));
   m = std::max(m, ws_route_bwd(d));
   return m + 256;
@@ -600,25 +606,11 @@ int moe_dispatch_bwd(const moe_shape_t* shape, const void* dx_perm, const float*
   return MOE_OK;
 }
 
-int moe_route_bwd(const moe_shape_t* shape, const void* x, const void* w_router, const int32_t* topk_idx,
-                  const float* topk_prob, const float* dtopk_prob, void* dx, float* dw_router, float* dlogits,
-                  void* ws, size_t ws_bytes, void* stream) {
-  Dims d;
-  TRY(check_shape(shape, &d));
-  REQUIRE_PTR(x);
-  REQUIRE_PTR(w_router);
-  REQUIRE_PTR(topk_idx);
-  REQUIRE_PTR(topk_prob);
-  REQUIRE_PTR(dtopk_prob);
-  REQUIRE_PTR(dx);
-  REQUIRE_PTR(dw_router);
-  REQUIRE_PTR(dlogits);
-  REQUIRE_PTR(ws);
-  if (ws_bytes < ws_route_bwd(d)) return MOE_ERR_WORKSPACE;
-  Ctx c;
-  TRY(get_ctx(stream, &c));
+// dx[T, Din] += dz . w_router and dw_router = dz^T . x, from dz [T, E] fp32 and
+// (bf16 inputs) its bf16 copy at the start of the workspace.
+static int router_grad_gemms(const Ctx& c, const Dims& d, const void* x, const void* w_router, const float* dlogits,
+                      void* dx, float* dw_router, void* ws) {
   void* dz16 = d.dt == DType::BF16 ? ws : nullptr;
-  TRY_CUDA(launch_route_dz(c, topk_idx, topk_prob, dtopk_prob, d.T, d.E, d.K, dlogits, dz16));
   // dx += dz . w_router   (M = T, N = Din, K = E)
   GemmDesc a;
   a.group = Group::Dense;
@@ -688,6 +680,97 @@ int moe_route_bwd(const moe_shape_t* shape, const void* x, const void* w_router,
   }
   TRY_CUDA(gemm(c, b, "router_wgrad_tc", "router_wgrad_simt"));
   return MOE_OK;
+}
+
+
+int moe_route_bwd(const moe_shape_t* shape, const void* x, const void* w_router, const int32_t* topk_idx,
+                  const float* topk_prob, const float* dtopk_prob, void* dx, float* dw_router, float* dlogits,
+                  void* ws, size_t ws_bytes, void* stream) {
+  Dims d;
+  TRY(check_shape(shape, &d));
+  REQUIRE_PTR(x);
+  REQUIRE_PTR(w_router);
+  REQUIRE_PTR(topk_idx);
+  REQUIRE_PTR(topk_prob);
+  REQUIRE_PTR(dtopk_prob);
+  REQUIRE_PTR(dx);
+  REQUIRE_PTR(dw_router);
+  REQUIRE_PTR(dlogits);
+  REQUIRE_PTR(ws);
+  if (ws_bytes < ws_route_bwd(d)) return MOE_ERR_WORKSPACE;
+  Ctx c;
+  TRY(get_ctx(stream, &c));
+  void* dz16 = d.dt == DType::BF16 ? ws : nullptr;
+  TRY_CUDA(launch_route_dz(c, topk_idx, topk_prob, dtopk_prob, d.T, d.E, d.K, dlogits, dz16));
+  return router_grad_gemms(c, d, x, w_router, dlogits, dx, dw_router, ws);
+}
+
+int moe_route_sigmoid(const moe_shape_t* shape, const void* x, const void* w_router, const float* expert_bias,
+                      float aux_coef, float* logits, int32_t* topk_idx, float* topk_prob, float* aux_f,
+                      float* aux_loss, void* ws, size_t ws_bytes, void* stream) {
+  Dims d;
+  TRY(check_shape(shape, &d));
+  REQUIRE_PTR(x);
+  REQUIRE_PTR(w_router);
+  OPTIONAL_PTR(expert_bias);
+  REQUIRE_PTR(logits);
+  REQUIRE_PTR(topk_idx);
+  REQUIRE_PTR(topk_prob);
+  REQUIRE_PTR(aux_f);
+  REQUIRE_PTR(aux_loss);
+  REQUIRE_PTR(ws);
+  if (ws_bytes < ws_route_sigmoid(d)) return MOE_ERR_WORKSPACE;
+  if (!(aux_coef == aux_coef)) return MOE_ERR_SHAPE;
+  Ctx c;
+  TRY(get_ctx(stream, &c));
+  GemmDesc g;
+  g.group = Group::Dense;
+  g.epi = Epi::StoreBias;  // with no bias: the instantiated fp32-output router GEMM
+  g.M = d.T;
+  g.N = d.E;
+  g.K = d.Din;
+  g.A = x;
+  g.a_type = d.dt;
+  g.sa_m = d.Din;
+  g.sa_k = 1;
+  g.B = w_router;
+  g.b_type = d.dt;
+  g.sb_n = d.Din;
+  g.sb_k = 1;
+  g.C = logits;
+  g.c_type = DType::F32;
+  g.ldc = d.E;
+  TRY_CUDA(gemm(c, g, "router_gemm_tc", "router_gemm_simt"));
+  TRY_CUDA(launch_route_sigmoid_select(c, logits, expert_bias, d.T, d.S, d.GBS, d.E, d.K, aux_coef, topk_idx,
+                                       topk_prob, aux_f, aux_loss, ws));
+  return MOE_OK;
+}
+
+int moe_route_sigmoid_bwd(const moe_shape_t* shape, const void* x, const void* w_router, const float* logits,
+                          const int32_t* topk_idx, const float* topk_prob, const float* dtopk_prob,
+                          const float* aux_f, float aux_coef, float aux_grad, void* dx, float* dw_router,
+                          float* dlogits, void* ws, size_t ws_bytes, void* stream) {
+  Dims d;
+  TRY(check_shape(shape, &d));
+  REQUIRE_PTR(x);
+  REQUIRE_PTR(w_router);
+  REQUIRE_PTR(logits);
+  REQUIRE_PTR(topk_idx);
+  REQUIRE_PTR(topk_prob);
+  REQUIRE_PTR(dtopk_prob);
+  REQUIRE_PTR(aux_f);
+  REQUIRE_PTR(dx);
+  REQUIRE_PTR(dw_router);
+  REQUIRE_PTR(dlogits);
+  REQUIRE_PTR(ws);
+  if (ws_bytes < ws_route_bwd(d)) return MOE_ERR_WORKSPACE;
+  if (!(aux_coef == aux_coef) || !(aux_grad == aux_grad)) return MOE_ERR_SHAPE;
+  Ctx c;
+  TRY(get_ctx(stream, &c));
+  void* dz16 = d.dt == DType::BF16 ? ws : nullptr;
+  TRY_CUDA(launch_route_dz_sigmoid(c, logits, topk_idx, topk_prob, dtopk_prob, aux_f, d.T, d.S, d.GBS, d.E, d.K,
+                                   aux_coef, aux_grad, dlogits, dz16));
+  return router_grad_gemms(c, d, x, w_router, dlogits, dx, dw_router, ws);
 }
 
 int moe_latent_proj(const moe_shape_t* shape, int32_t n_in, int32_t n_out, const void* in, const void* w,

@@ -58,6 +58,21 @@ cudaError_t launch_route_dz(const Ctx& c, const int32_t* idx, const float* prob,
                             int E, int K, float* dz, void* dz_bf16);
 
 // ---------------------------------------------------------------------------
+// router_sigmoid.cu
+// ---------------------------------------------------------------------------
+size_t route_sigmoid_fwd_ws_bytes(int64_t T, int64_t S, int64_t GBS, int E);
+// idx/prob [T, K] from the sigmoid scores of logits [T, E] (bias [E] for the
+// choice only, may be NULL), f [GBS, E] and loss [1] of the sequence-level
+// balance loss.
+cudaError_t launch_route_sigmoid_select(const Ctx& c, const float* logits, const float* bias, int64_t T, int64_t S,
+                                        int64_t GBS, int E, int K, float coef, int32_t* idx, float* prob,
+                                        float* f_out, float* loss, void* ws);
+// dz [T, E] fp32 (fully written) and optionally a bf16 copy.
+cudaError_t launch_route_dz_sigmoid(const Ctx& c, const float* logits, const int32_t* idx, const float* prob,
+                                    const float* dprob, const float* f, int64_t T, int64_t S, int64_t GBS, int E,
+                                    int K, float coef, float aux_grad, float* dz, void* dz16);
+
+// ---------------------------------------------------------------------------
 // permute.cu
 // ---------------------------------------------------------------------------
 size_t perm_workspace_bytes(int64_t TK, int E);

@@ -18,9 +18,21 @@ def _dt(dtype: str):
 
 
 class MoeLayer:
-    """All buffers of one layer step for one shape, allocated once on ``device``."""
+    """All buffers of one layer step for one shape, allocated once on ``device``.
 
-    def __init__(self, S, GBS, K, D, E, F, dtype="bf16", H=0, device="cuda"):
+    ``router="softmax"`` routes with softmax + renormalised top-K;
+    ``router="sigmoid"`` with sigmoid scores, a selection-only expert bias and
+    the sequence-level balance loss (coefficient ``aux_coef``; its gradient
+    enters the backward pass scaled by ``aux_grad``), Sec. 5.2.
+    """
+
+    def __init__(self, S, GBS, K, D, E, F, dtype="bf16", H=0, device="cuda", router="softmax", aux_coef=1e-4,
+                 aux_grad=1.0):
+        if router not in ("softmax", "sigmoid"):
+            raise ValueError(f"unknown router {router!r}")
+        self.router = router
+        self.aux_coef = float(aux_coef)
+        self.aux_grad = float(aux_grad)
         self.shape = abi.MoeShape.of(S, GBS, K, D, E, F, dtype, H)
         self.T = T = S * GBS
         self.TK = TK = T * K
@@ -37,6 +49,7 @@ class MoeLayer:
         self.w1 = e(E, 2 * F, D)
         self.w2 = e(E, D, F)
         self.bias = None
+        self.expert_bias = torch.zeros(E, dtype=f32, device=dev) if router == "sigmoid" else None
         self.w_down = e(D, H) if H else None
         self.w_upp = e(H, D) if H else None
         # forward
@@ -44,6 +57,8 @@ class MoeLayer:
         self.logits = e(T, E, d=f32)
         self.topk_idx = e(T, K, d=i32)
         self.topk_prob = e(T, K, d=f32)
+        self.aux_f = e(GBS, E, d=f32) if router == "sigmoid" else None
+        self.aux_loss = e(4, d=f32) if router == "sigmoid" else None
         self.x_lat = e(T, D) if H else None
         self.expert_offsets = e(E + 1, d=i32)
         self.row_of_slot = e(TK, d=i32)
@@ -89,12 +104,18 @@ class MoeLayer:
             self.bias = inputs["bias"].to(self.x.device, non_blocking=True).contiguous()
         else:
             self.bias = None
+        if self.router == "sigmoid" and inputs.get("expert_bias") is not None:
+            self.expert_bias.copy_(inputs["expert_bias"], non_blocking=True)
 
     # ------------------------------------------------------------------
     def forward(self, stream=None):
         s = self.shape
-        abi.moe_route(s, self.x, self.w_router, self.bias, self.logits, self.topk_idx, self.topk_prob, self.ws,
-                      stream)
+        if self.router == "sigmoid":
+            abi.moe_route_sigmoid(s, self.x, self.w_router, self.expert_bias, self.aux_coef, self.logits,
+                                  self.topk_idx, self.topk_prob, self.aux_f, self.aux_loss, self.ws, stream)
+        else:
+            abi.moe_route(s, self.x, self.w_router, self.bias, self.logits, self.topk_idx, self.topk_prob, self.ws,
+                          stream)
         xd = self.x
         if self.H:
             abi.moe_latent_proj(s, self.H, self.D, self.x, self.w_down, self.x_lat, self.ws, stream)
@@ -127,8 +148,13 @@ class MoeLayer:
                                     self.dw_down, self.ws, stream)
         else:
             abi.moe_dispatch_bwd(s, self.dx_perm, self.dprob_perm, self.row_of_slot, self.dx, self.dprob, stream)
-        abi.moe_route_bwd(s, self.x, self.w_router, self.topk_idx, self.topk_prob, self.dprob, self.dx,
-                          self.dw_router, self.dlogits, self.ws, stream)
+        if self.router == "sigmoid":
+            abi.moe_route_sigmoid_bwd(s, self.x, self.w_router, self.logits, self.topk_idx, self.topk_prob,
+                                      self.dprob, self.aux_f, self.aux_coef, self.aux_grad, self.dx, self.dw_router,
+                                      self.dlogits, self.ws, stream)
+        else:
+            abi.moe_route_bwd(s, self.x, self.w_router, self.topk_idx, self.topk_prob, self.dprob, self.dx,
+                              self.dw_router, self.dlogits, self.ws, stream)
         return self.dx
 
     def step(self, stream=None):

@@ -25,6 +25,8 @@ Public layouts (row-major):
   w_down  [D, H]        LatentMoE down-projection, x_lat = x . w_down^T
   w_upp   [H, D]        LatentMoE up-projection,   out = y_lat . w_upp^T
   bias    [E] float32   per-expert logit bias (skewed workload only)
+  expert_bias [E] float32  selection-only bias of the sigmoid router
+                        (``make_expert_bias``, drawn separately)
   dy      [T, D]        upstream gradient (LatentMoE: [T, H])
 """
 from __future__ import annotations
@@ -92,6 +94,13 @@ def get(name: str) -> Workload:
 def skew_bias_values(E: int) -> torch.Tensor:
     """Per-expert logit bias of the skewed workload: b_e = 3 * ln(1/(e+1)), e 0-based, in float32."""
     return torch.tensor([3.0 * math.log(1.0 / (e + 1)) for e in range(E)], dtype=torch.float32)
+
+
+def make_expert_bias(E: int, seed: int, std: float = 0.05) -> torch.Tensor:
+    """Expert bias [E] float32 for the sigmoid router, N(0, std) from its own
+    generator (seed + 7919), so it leaves the ``make_inputs`` stream alone."""
+    g = torch.Generator().manual_seed(int(seed) + 7919)
+    return torch.randn(E, generator=g, dtype=torch.float32) * std
 
 
 def _storage(dtype: str) -> torch.dtype:
