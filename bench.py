@@ -66,6 +66,9 @@ def kernel_work(name: str, w: synth.Workload, T: int) -> tuple[str, float]:
         "combine_bwd": (T + 2 * TK) * D * bx + 12 * TK,
         "dispatch_bwd": (TK + T) * D * bx + 8 * TK,
         "route_dz": T * K * 12 + T * E * 6,
+        "select_sigmoid": T * E * 4 + T * K * 8,
+        "balance_finalize": 0.0,
+        "route_dz_sigmoid": T * E * 4 + T * K * 12 + T * E * 6,
         "swiglu_bwd": 5.0 * TK * F * bx,
         "pack_w1": 0.0,
     }
@@ -254,6 +257,8 @@ def main() -> None:
     ap.add_argument("--cpu-budget", type=float, default=15.0, help="seconds of CPU work for cpu_baseline")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=10)
+    ap.add_argument("--router", default="softmax", choices=["softmax", "sigmoid"],
+                    help="softmax top-K, or sigmoid scores + expert bias + sequence-level balance loss (Sec. 5.2)")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
     w = synth.get(args.workload)
@@ -279,7 +284,9 @@ def main() -> None:
 
     T = w.T
     inputs = synth.make_inputs(w, seed=rank_seed(w, rank))      # each rank its own tokens
-    L = MoeLayer(w.S, w.GBS, w.K, w.D, w.E, w.F, w.dtype, w.H)
+    if args.router == "sigmoid":
+        inputs["expert_bias"] = synth.make_expert_bias(w.E, rank_seed(w, rank))
+    L = MoeLayer(w.S, w.GBS, w.K, w.D, w.E, w.F, w.dtype, w.H, router=args.router)
     L.load(inputs)
     stream = torch.cuda.current_stream()
     flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device="cuda")
@@ -293,30 +300,40 @@ def main() -> None:
     torch.cuda.synchronize()
     assert abi.moe_check_device_status() == 0
 
-    # ---- timed region: K steps, L2 flushed before each (outside the events)
-    ev_s = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
-    ev_e = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
-    abi.moe_prof_reset()
-    abi.moe_prof_enable(True)
-    n0 = abi.moe_launch_count()
+    def timed_steps(kernel_events: bool):
+        """K steps, L2 flushed before each (outside the step events).  With
+        kernel_events the library also brackets every kernel with CUDA events
+        on its stream (per-kernel durations for the roofline); those records
+        sit between the kernels, so the headline step time comes from the pass
+        without them."""
+        ev_s = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+        ev_e = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+        abi.moe_prof_reset()
+        abi.moe_prof_enable(kernel_events)
+        n0 = abi.moe_launch_count()
+        barrier()
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        for i in range(args.steps):
+            flush.zero_()
+            ev_s[i].record(stream)
+            L.step()
+            ev_e[i].record(stream)
+        torch.cuda.synchronize()
+        barrier()
+        wall = time.perf_counter() - t0
+        launches = (abi.moe_launch_count() - n0) // args.steps
+        abi.moe_prof_enable(False)
+        prof = abi.moe_prof_read() if kernel_events else {}
+        step_ms = sum(s.elapsed_time(e) for s, e in zip(ev_s, ev_e)) / args.steps
+        return step_ms, wall, launches, prof
+
     clocks = ClockSampler(local)
-    barrier()
-    torch.cuda.synchronize()
-    t0 = time.perf_counter()
-    for i in range(args.steps):
-        flush.zero_()
-        ev_s[i].record(stream)
-        L.step()
-        ev_e[i].record(stream)
-    torch.cuda.synchronize()
-    barrier()
-    wall = time.perf_counter() - t0
+    step_ms, wall, launches, _ = timed_steps(kernel_events=False)
     clk = clocks.stop()
-    launches = (abi.moe_launch_count() - n0) // args.steps
-    abi.moe_prof_enable(False)
-    prof = abi.moe_prof_read()
-    step_ms = sum(s.elapsed_time(e) for s, e in zip(ev_s, ev_e)) / args.steps
     t_max = max_over_ranks(step_ms, world, "cuda")
+    assert abi.moe_check_device_status() == 0
+    step_ms_ev, _, _, prof = timed_steps(kernel_events=True)
     assert abi.moe_check_device_status() == 0
 
     # ---- end to end through the public API with host buffers
@@ -386,7 +403,7 @@ def main() -> None:
               for k, v in sorted(kernels.items(), key=lambda kv: -kv[1]["ms_per_step"])}
 
     cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+    if rank == 0 and world == 1 and not args.no_cpu_baseline and args.router == "softmax":
         cpu = cpu_baseline(w, args.cpu_budget)
 
     if rank == 0:
@@ -395,7 +412,8 @@ def main() -> None:
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": t_max, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
             "config": {"workload": w.name, "T": T, "S": w.S, "GBS": w.GBS, "D": w.D, "E": w.E, "K": w.K, "F": w.F,
-                       "H": w.H, "seed": w.seed, "parallelism": f"replicas x{world}, each rank its own tokens",
+                       "H": w.H, "seed": w.seed, "router": args.router,
+                       "parallelism": f"replicas x{world}, each rank its own tokens",
                        "l2": "256 MiB buffer written before every timed step (outside the step events); "
                              "the step also touches ~3 GB > 129 MB L2"},
             "roofline": roof,
@@ -407,6 +425,7 @@ def main() -> None:
             "gpu_launches_per_step": launches,
             "clocks": clk,
             "wall_s_timed_region": wall,
+            "ms_per_step_kernel_events_pass": round(step_ms_ev, 4),
             "kernels": detail,
         }
         print(json.dumps(line), flush=True)

@@ -1,92 +1,70 @@
-// Router kernels: warp-per-token top-K with renormalised probabilities, and
+// Router kernels: top-K with renormalised probabilities, and
 // the router backward dz = p (dp - sum_k p_k dp_k) on the chosen set.
 #include <math_constants.h>
 
 #include "common.cuh"
 #include "launch.h"
+#include "select.cuh"
 
 namespace moe {
 
-// One warp per token.  Lane l holds logits l, l + 32, ... (VPL per lane).  K
-// rounds of a warp arg-max pick the largest remaining logit, ties to the lower
-// expert index (reading R2); NaN is treated as -inf.  The probabilities are
-// exp(z_k - z_max) normalised over the K chosen logits, which equals the full
-// softmax renormalised over the chosen set (reading R1).
-template <int VPL>
+struct Identity {
+  __device__ __forceinline__ float operator()(float z) const { return z; }
+};
+
+// Four threads per token (select.cuh): the K largest logits, ties to the lower
+// expert index (reading R2), NaN as -inf, ordered by descending logit.  The
+// probabilities are exp(z_k - z_max) normalised over the K chosen logits,
+// which equals the full softmax renormalised over the chosen set (reading R1).
+template <int KM>
 __global__ void __launch_bounds__(256) topk_kernel(const float* __restrict__ logits, int64_t T, int E, int K,
-                                                   int32_t* __restrict__ idx, float* __restrict__ prob) {
-  const int lane = threadIdx.x & 31;
-  const int64_t t = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
-  if (t >= T) return;
-  const float* row = logits + t * E;
-  float v[VPL];
-  unsigned alive = 0;
-#pragma unroll
-  for (int j = 0; j < VPL; ++j) {
-    const int e = lane + 32 * j;
-    float z = -CUDART_INF_F;
-    if (e < E) {
-      z = __ldg(row + e);
-      if (z != z) z = -CUDART_INF_F;
-      alive |= 1u << j;
-    }
-    v[j] = z;
-  }
-  float sel_v[kMaxK];
-  int sel_i[kMaxK];
-#pragma unroll
-  for (int k = 0; k < kMaxK; ++k) {
-    if (k < K) {
-      float bv = -CUDART_INF_F;
-      int bi = 0x7fffffff;
-#pragma unroll
-      for (int j = 0; j < VPL; ++j) {
-        const int e = lane + 32 * j;
-        if ((alive >> j) & 1u) {
-          if (v[j] > bv || (v[j] == bv && e < bi)) { bv = v[j]; bi = e; }
-        }
-      }
-#pragma unroll
-      for (int off = 16; off > 0; off >>= 1) {
-        const float ov = __shfl_xor_sync(0xffffffffu, bv, off);
-        const int oi = __shfl_xor_sync(0xffffffffu, bi, off);
-        if (ov > bv || (ov == bv && oi < bi)) { bv = ov; bi = oi; }
-      }
-      if (lane == (bi & 31)) alive &= ~(1u << (bi >> 5));
-      sel_v[k] = bv;
-      sel_i[k] = bi;
-    }
-  }
-  const float zmax = sel_v[0];
-  float w[kMaxK];
+                                                   int tpb, int32_t* __restrict__ idx, float* __restrict__ prob) {
+  extern __shared__ __align__(16) float zs[];  // [tpb][E]
+  const int tid = threadIdx.x;
+  const int64_t t0 = (int64_t)blockIdx.x * tpb;
+  const int n = (int)min((int64_t)tpb, T - t0);
+  sel::stage_rows(logits + t0 * E, zs, n * E, Identity());
+  __syncthreads();
+  const int q = tid >> 2, r = tid & 3;
+  const bool active = q < n;
+  uint64_t win[KM];
+  float unused;
+  sel::quad_topk<KM>(zs + (int64_t)q * E, nullptr, E, K, r, q, active, win, &unused);
+  if (!active) return;
+  const float zmax = sel::unpack_key(win[0]);
+  float w[KM];
   float sum = 0.f;
 #pragma unroll
-  for (int k = 0; k < kMaxK; ++k) {
+  for (int k = 0; k < KM; ++k) {
+    w[k] = 0.f;
     if (k < K) {
-      w[k] = expf(sel_v[k] - zmax);
+      w[k] = expf(sel::unpack_key(win[k]) - zmax);
       sum += w[k];
     }
   }
   const float inv = 1.0f / sum;
+  const int64_t o = (t0 + q) * K;
 #pragma unroll
-  for (int k = 0; k < kMaxK; ++k) {
-    if (k < K && lane == k) {
-      idx[t * K + k] = sel_i[k];
-      prob[t * K + k] = w[k] * inv;
+  for (int k = 0; k < KM; ++k) {
+    if (k < K && (k & 3) == r) {
+      idx[o + k] = sel::unpack_e(win[k]);
+      prob[o + k] = w[k] * inv;
     }
   }
 }
 
 cudaError_t launch_topk(const Ctx& c, const float* logits, int64_t T, int E, int K, int32_t* idx, float* prob) {
   if (T == 0) return cudaSuccess;
-  const int warps = 8;
-  dim3 grid((unsigned)((T + warps - 1) / warps)), block(32 * warps);
+  const int tpb = sel::tokens_per_block(E);
+  const dim3 grid((unsigned)((T + tpb - 1) / tpb));
+  const size_t smem = (size_t)tpb * E * 4;
   KernelScope ks("topk", c.stream);
-  const int vpl = (E + 31) / 32;
-  if (vpl <= 1) topk_kernel<1><<<grid, block, 0, c.stream>>>(logits, T, E, K, idx, prob);
-  else if (vpl <= 2) topk_kernel<2><<<grid, block, 0, c.stream>>>(logits, T, E, K, idx, prob);
-  else if (vpl <= 4) topk_kernel<4><<<grid, block, 0, c.stream>>>(logits, T, E, K, idx, prob);
-  else topk_kernel<8><<<grid, block, 0, c.stream>>>(logits, T, E, K, idx, prob);
+  switch (sel::k_bound(K)) {
+    case 2: topk_kernel<2><<<grid, 4 * tpb, smem, c.stream>>>(logits, T, E, K, tpb, idx, prob); break;
+    case 4: topk_kernel<4><<<grid, 4 * tpb, smem, c.stream>>>(logits, T, E, K, tpb, idx, prob); break;
+    case 8: topk_kernel<8><<<grid, 4 * tpb, smem, c.stream>>>(logits, T, E, K, tpb, idx, prob); break;
+    default: topk_kernel<16><<<grid, 4 * tpb, smem, c.stream>>>(logits, T, E, K, tpb, idx, prob); break;
+  }
   return cudaGetLastError();
 }
 

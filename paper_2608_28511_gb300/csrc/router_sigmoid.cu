@@ -5,149 +5,153 @@
 //   p_k = s_k / sum_{j in S} s_j;
 //   per sequence g of S tokens: f_gi = E / (K S) #{t in g : i chosen},
 //   P_gi = mean over t in g of s_ti / sum_j s_tj, L = coef / GBS sum_g,i f_gi P_gi.
-// All reductions run in a fixed order, so results are bit-reproducible.
+// All reductions run in a fixed order (integer atomics only), so results are
+// bit-reproducible.
 #include <math_constants.h>
 
 #include "common.cuh"
 #include "launch.h"
+#include "select.cuh"
 
 namespace moe {
 
 namespace {
 
-constexpr int kTokChunk = 256;  // tokens per partial sum of the balance statistics
-
-__device__ __forceinline__ float sigmoidf_(float z) { return 1.0f / (1.0f + __expf(-z)); }
-
-// One warp per token: scores, the biased choice, gate values and the token's
-// score sum (for the balance statistics).
-template <int VPL>
-__global__ void __launch_bounds__(256) topk_sigmoid_kernel(const float* __restrict__ logits,
-                                                           const float* __restrict__ bias, int64_t T, int E, int K,
-                                                           int32_t* __restrict__ idx, float* __restrict__ prob,
-                                                           float* __restrict__ rowsum) {
-  const int lane = threadIdx.x & 31;
-  const int64_t t = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
-  if (t >= T) return;
-  const float* row = logits + t * E;
-  float s[VPL], key[VPL];
-  unsigned alive = 0;
-  float ssum = 0.f;
-#pragma unroll
-  for (int j = 0; j < VPL; ++j) {
-    const int e = lane + 32 * j;
-    s[j] = 0.f;
-    key[j] = -CUDART_INF_F;
-    if (e < E) {
-      s[j] = sigmoidf_(__ldg(row + e));
-      key[j] = s[j] + (bias ? __ldg(bias + e) : 0.f);
-      if (key[j] != key[j]) key[j] = -CUDART_INF_F;
-      alive |= 1u << j;
-      ssum += s[j];
-    }
-  }
-#pragma unroll
-  for (int off = 16; off > 0; off >>= 1) ssum += __shfl_xor_sync(0xffffffffu, ssum, off);
-  int sel_i[kMaxK];
-  float sel_s[kMaxK];
-  float gsum = 0.f;
-#pragma unroll
-  for (int k = 0; k < kMaxK; ++k) {
-    if (k < K) {
-      float bv = -CUDART_INF_F, bs = 0.f;
-      int bi = 0x7fffffff;
-#pragma unroll
-      for (int j = 0; j < VPL; ++j) {
-        const int e = lane + 32 * j;
-        if ((alive >> j) & 1u) {
-          if (key[j] > bv || (key[j] == bv && e < bi)) { bv = key[j]; bi = e; bs = s[j]; }
-        }
-      }
-#pragma unroll
-      for (int off = 16; off > 0; off >>= 1) {
-        const float ov = __shfl_xor_sync(0xffffffffu, bv, off);
-        const int oi = __shfl_xor_sync(0xffffffffu, bi, off);
-        const float os = __shfl_xor_sync(0xffffffffu, bs, off);
-        if (ov > bv || (ov == bv && oi < bi)) { bv = ov; bi = oi; bs = os; }
-      }
-      if (lane == (bi & 31)) alive &= ~(1u << (bi >> 5));
-      sel_i[k] = bi;
-      sel_s[k] = bs;
-      gsum += bs;
-    }
-  }
-  const float inv = 1.0f / gsum;
-#pragma unroll
-  for (int k = 0; k < kMaxK; ++k) {
-    if (k < K && lane == k) {
-      idx[t * K + k] = sel_i[k];
-      prob[t * K + k] = sel_s[k] * inv;
-    }
-  }
-  if (lane == 0) rowsum[t] = ssum;
+int64_t select_chunks(int64_t S, int E) {
+  return (S + sel::tokens_per_block(E) - 1) / sel::tokens_per_block(E);
 }
 
-// Partial balance statistics: block (g, chunk) sums, for every expert, the
-// normalised scores and the choice counts of up to kTokChunk tokens of
-// sequence g, in token order.
-__global__ void __launch_bounds__(256) aux_partial_kernel(const float* __restrict__ logits,
-                                                          const float* __restrict__ rowsum,
-                                                          const int32_t* __restrict__ idx, int64_t S, int E, int K,
-                                                          int nchunk, float* __restrict__ psum,
-                                                          int32_t* __restrict__ pcnt) {
-  const int g = blockIdx.y, ch = blockIdx.x;
-  const int64_t t0 = (int64_t)g * S + (int64_t)ch * kTokChunk;
-  const int64_t t1 = min((int64_t)g * S + S, t0 + kTokChunk);
-  __shared__ int32_t sidx[kTokChunk * kMaxK];
-  __shared__ float srs[kTokChunk];
-  for (int64_t i = threadIdx.x; i < (t1 - t0) * K; i += blockDim.x) sidx[i] = idx[t0 * K + i];
-  for (int64_t i = threadIdx.x; i < t1 - t0; i += blockDim.x) srs[i] = rowsum[t0 + i];
+__device__ __forceinline__ float sigmoidf_(float z) { return __frcp_rn(1.0f + __expf(-z)); }
+
+struct SigmoidOp {
+  __device__ __forceinline__ float operator()(float z) const { return sigmoidf_(z); }
+};
+
+// Block (chunk ch of sequence g): stages the scores s = sigmoid(z) of its
+// tokens, chooses each token's K experts by s + b (four threads per token),
+// writes idx and the gate values s_k / sum over the chosen of s, then adds up,
+// per expert, the normalised scores (in token order) and the choice counts of
+// its tokens: one partial per (sequence, chunk).
+template <int KM>
+__global__ void __launch_bounds__(256) select_sigmoid_kernel(
+    const float* __restrict__ logits, const float* __restrict__ bias, int64_t S, int E, int K, int tpb, int nch,
+    int32_t* __restrict__ idx, float* __restrict__ prob, float* __restrict__ psum, int32_t* __restrict__ pcnt,
+    uint32_t* __restrict__ ticket) {
+  extern __shared__ __align__(16) float sm[];
+  float* zs = sm;                                   // [tpb][E] scores
+  float* bs = zs + tpb * E;                         // [E]
+  float* inv = bs + E;                              // [tpb]
+  int* cnt = reinterpret_cast<int*>(inv + tpb);     // [E]
+  const int tid = threadIdx.x, ch = blockIdx.x, g = blockIdx.y;
+  const int64_t t0 = (int64_t)g * S + (int64_t)ch * tpb;
+  const int n = (int)min((int64_t)tpb, S - (int64_t)ch * tpb);
+  sel::stage_rows(logits + t0 * E, zs, n * E, SigmoidOp());
+  for (int e = tid; e < E; e += blockDim.x) {
+    bs[e] = bias ? __ldg(bias + e) : 0.f;
+    cnt[e] = 0;
+  }
+  if (ch == 0 && g == 0 && tid == 0) *ticket = 0u;  // for the finalize kernel that follows
   __syncthreads();
-  for (int e = threadIdx.x; e < E; e += blockDim.x) {
+  const int q = tid >> 2, r = tid & 3;
+  const bool active = q < n;
+  const float* row = zs + (int64_t)q * E;
+  uint64_t win[KM];
+  float ssum;
+  sel::quad_topk<KM>(row, bs, E, K, r, q, active, win, &ssum);
+  if (active) {
+    float gsum = 0.f;
+#pragma unroll
+    for (int k = 0; k < KM; ++k)
+      if (k < K) gsum += row[sel::unpack_e(win[k])];
+    const float ginv = __frcp_rn(gsum);
+    const int64_t o = (t0 + q) * K;
+#pragma unroll
+    for (int k = 0; k < KM; ++k) {
+      if (k < K && (k & 3) == r) {
+        const int e = sel::unpack_e(win[k]);
+        idx[o + k] = e;
+        prob[o + k] = row[e] * ginv;
+        atomicAdd(cnt + e, 1);
+      }
+    }
+    if (r == 0) inv[q] = __frcp_rn(ssum);
+  }
+  __syncthreads();
+  const int64_t o = ((int64_t)g * nch + ch) * E;
+  for (int e = tid; e < E; e += blockDim.x) {
     float acc = 0.f;
-    int cnt = 0;
-    for (int64_t t = t0; t < t1; ++t) {
-      acc += sigmoidf_(logits[t * E + e]) / srs[t - t0];
-      for (int k = 0; k < K; ++k) cnt += sidx[(t - t0) * K + k] == e;
-    }
-    const int64_t o = ((int64_t)g * nchunk + ch) * E + e;
-    psum[o] = acc;
-    pcnt[o] = cnt;
+#pragma unroll 8
+    for (int t = 0; t < n; ++t) acc += zs[t * E + e] * inv[t];
+    psum[o + e] = acc;
+    pcnt[o + e] = cnt[e];
   }
 }
 
-// f [GBS, E] and the loss: one block, chunks and then (g, e) summed in order.
-__global__ void __launch_bounds__(256) aux_finalize_kernel(const float* __restrict__ psum,
-                                                           const int32_t* __restrict__ pcnt, int GBS, int64_t S,
-                                                           int E, int K, int nchunk, float coef,
-                                                           float* __restrict__ f_out, float* __restrict__ loss) {
-  __shared__ float red[256];
-  float part = 0.f;
-  for (int i = threadIdx.x; i < GBS * E; i += blockDim.x) {
-    const int g = i / E, e = i % E;
-    float P = 0.f;
-    int64_t cnt = 0;
-    for (int ch = 0; ch < nchunk; ++ch) {
-      const int64_t o = ((int64_t)g * nchunk + ch) * E + e;
+// f [GBS, E] and the loss.  Block (expert tile of 32, sequence g): warp w adds
+// chunks w, w + 8, ...; warp 0 combines the 8 warps in order, writes f and the
+// tile's sum of f P; the last block to finish adds the tiles in order.
+__global__ void __launch_bounds__(256) balance_finalize_kernel(const float* __restrict__ psum,
+                                                               const int32_t* __restrict__ pcnt, int64_t S, int E,
+                                                               int K, int nch, float coef, int GBS,
+                                                               float* __restrict__ f_out, float* __restrict__ tile_sum,
+                                                               uint32_t* __restrict__ ticket,
+                                                               float* __restrict__ loss) {
+  __shared__ float rp[8][32];
+  __shared__ int rc[8][32];
+  const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+  const int e = blockIdx.x * 32 + l, g = blockIdx.y;
+  float P = 0.f;
+  int c = 0;
+  if (e < E) {
+    for (int ch = w; ch < nch; ch += 8) {
+      const int64_t o = ((int64_t)g * nch + ch) * E + e;
       P += psum[o];
-      cnt += pcnt[o];
+      c += pcnt[o];
     }
-    const float f = (float)((double)E / ((double)K * (double)S) * (double)cnt);
-    f_out[i] = f;
-    part += f * (P / (float)S);
   }
-  red[threadIdx.x] = part;
+  rp[w][l] = P;
+  rc[w][l] = c;
   __syncthreads();
-  for (int off = 128; off > 0; off >>= 1) {
-    if (threadIdx.x < off) red[threadIdx.x] += red[threadIdx.x + off];
-    __syncthreads();
+  if (w != 0) return;
+  P = 0.f;
+  c = 0;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    P += rp[i][l];
+    c += rc[i][l];
   }
-  if (threadIdx.x == 0) loss[0] = coef / (float)GBS * red[0];
+  float prod = 0.f;
+  if (e < E) {
+    const float f = (float)((double)E / ((double)K * (double)S) * (double)c);
+    f_out[(int64_t)g * E + e] = f;
+    prod = f * (P / (float)S);
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) prod += __shfl_xor_sync(0xffffffffu, prod, off);
+  const int nblk = gridDim.x * gridDim.y;
+  unsigned last = 0;
+  if (l == 0) {
+    tile_sum[blockIdx.y * gridDim.x + blockIdx.x] = prod;
+    __threadfence();
+    last = atomicAdd(ticket, 1u) == (unsigned)(nblk - 1);
+  }
+  last = __shfl_sync(0xffffffffu, last, 0);
+  if (!last) return;
+  __threadfence();
+  float tot = 0.f;
+  for (int i = l; i < nblk; i += 32) tot += __ldcg(tile_sum + i);
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) tot += __shfl_xor_sync(0xffffffffu, tot, off);
+  if (l == 0) {
+    loss[0] = coef / (float)GBS * tot;
+    *ticket = 0u;
+  }
 }
 
-// One warp per token: gradient of the gate values of the chosen experts plus
-// aux_grad times the balance loss with respect to the logits (all E entries),
-// and its bf16 copy.
+// One warp per token; lane l holds experts l, l + 32, ...  Gradient of the
+// gate values of the chosen experts plus aux_grad times the balance loss with
+// respect to all E logits, and its bf16 copy.
+template <int VPL>
 __global__ void __launch_bounds__(256) route_dz_sigmoid_kernel(
     const float* __restrict__ logits, const int32_t* __restrict__ idx, const float* __restrict__ prob,
     const float* __restrict__ dprob, const float* __restrict__ f, int64_t T, int64_t S, int E, int K, float cscale,
@@ -155,23 +159,29 @@ __global__ void __launch_bounds__(256) route_dz_sigmoid_kernel(
   const int lane = threadIdx.x & 31;
   const int64_t t = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   if (t >= T) return;
-  const int64_t g = t / S;
   const float* row = logits + t * E;
-  const float* fg = f + g * E;
-  // score sum and sum_i c_i shat_i numerator over the whole row
+  const float* fg = f + (t / S) * E;
+  float s[VPL], c[VPL];
   float ssum = 0.f, csum = 0.f;
-  for (int e = lane; e < E; e += 32) {
-    const float sv = sigmoidf_(row[e]);
-    ssum += sv;
-    csum += cscale * fg[e] * sv;
+#pragma unroll
+  for (int j = 0; j < VPL; ++j) {
+    const int e = lane + 32 * j;
+    s[j] = 0.f;
+    c[j] = 0.f;
+    if (e < E) {
+      s[j] = sigmoidf_(__ldg(row + e));
+      c[j] = cscale * __ldg(fg + e);
+      ssum += s[j];
+      csum += c[j] * s[j];
+    }
   }
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) {
     ssum += __shfl_xor_sync(0xffffffffu, ssum, off);
     csum += __shfl_xor_sync(0xffffffffu, csum, off);
   }
-  const float cbar = csum / ssum;  // sum_i c_i shat_i
-  // gate path: chosen experts' scores, gate values and incoming gradients
+  const float rs = __frcp_rn(ssum);
+  const float cbar = csum * rs;  // sum_i c_i s_i / sum_i s_i
   int my_e = -1;
   float my_p = 0.f, my_dp = 0.f, my_s = 0.f;
   if (lane < K) {
@@ -179,7 +189,7 @@ __global__ void __launch_bounds__(256) route_dz_sigmoid_kernel(
     if (my_e >= 0 && my_e < E) {
       my_p = prob[t * K + lane];
       my_dp = dprob[t * K + lane];
-      my_s = sigmoidf_(row[my_e]);
+      my_s = sigmoidf_(__ldg(row + my_e));
     } else {
       set_error(err, kErrIndex);  // an out-of-range expert index contributes nothing
       my_e = -1;
@@ -191,62 +201,77 @@ __global__ void __launch_bounds__(256) route_dz_sigmoid_kernel(
     dot += __shfl_xor_sync(0xffffffffu, dot, off);
     gs += __shfl_xor_sync(0xffffffffu, gs, off);
   }
-  const float my_gate = (my_dp - dot) / gs;
-  for (int e0 = 0; e0 < E; e0 += 32) {
-    const int e = e0 + lane;
-    float gate = 0.f;
-    for (int k = 0; k < K; ++k) {
+  const float my_gate = (my_dp - dot) * __frcp_rn(gs);
+  float gate[VPL];
+#pragma unroll
+  for (int j = 0; j < VPL; ++j) gate[j] = 0.f;
+#pragma unroll
+  for (int k = 0; k < kMaxK; ++k) {
+    if (k < K) {
       const int ek = __shfl_sync(0xffffffffu, my_e, k);
       const float gk = __shfl_sync(0xffffffffu, my_gate, k);
-      if (ek == e) gate = gk;
+#pragma unroll
+      for (int j = 0; j < VPL; ++j)
+        if (ek == lane + 32 * j) gate[j] = gk;
     }
+  }
+#pragma unroll
+  for (int j = 0; j < VPL; ++j) {
+    const int e = lane + 32 * j;
     if (e < E) {
-      const float sv = sigmoidf_(row[e]);
-      const float ds = gate + (cscale * fg[e] - cbar) / ssum;
-      const float v = sv * (1.0f - sv) * ds;
+      const float v = s[j] * (1.0f - s[j]) * (gate[j] + (c[j] - cbar) * rs);
       dz[t * E + e] = v;
       if (dz16) dz16[t * E + e] = __float2bfloat16_rn(v);
     }
   }
 }
 
+size_t align256(size_t v) { return (v + 255) & ~size_t(255); }
+
 }  // namespace
 
 size_t route_sigmoid_fwd_ws_bytes(int64_t T, int64_t S, int64_t GBS, int E) {
-  const int64_t nchunk = (S + kTokChunk - 1) / kTokChunk;
-  return (size_t)T * 4 + (size_t)GBS * nchunk * E * 8 + 512;
+  (void)T;
+  const int64_t parts = GBS * select_chunks(S, E) * E;
+  const int64_t tiles = GBS * ((E + 31) / 32);
+  return align256(parts * 4) * 2 + align256(tiles * 4) + 256;
 }
 
 cudaError_t launch_route_sigmoid_select(const Ctx& c, const float* logits, const float* bias, int64_t T, int64_t S,
                                         int64_t GBS, int E, int K, float coef, int32_t* idx, float* prob,
                                         float* f_out, float* loss, void* ws) {
   if (T == 0) return cudaSuccess;
-  float* rowsum = static_cast<float*>(ws);
-  const int64_t nchunk = (S + kTokChunk - 1) / kTokChunk;
-  float* psum = rowsum + ((T + 63) / 64) * 64;
-  int32_t* pcnt = reinterpret_cast<int32_t*>(psum + GBS * nchunk * E);
+  const int tpb = sel::tokens_per_block(E);
+  const int64_t nch = select_chunks(S, E);
+  const int64_t parts = GBS * nch * E;
+  const int64_t tiles = GBS * ((E + 31) / 32);
+  char* base = static_cast<char*>(ws);
+  float* psum = reinterpret_cast<float*>(base);
+  int32_t* pcnt = reinterpret_cast<int32_t*>(base + align256(parts * 4));
+  float* tile_sum = reinterpret_cast<float*>(base + 2 * align256(parts * 4));
+  uint32_t* ticket = reinterpret_cast<uint32_t*>(base + 2 * align256(parts * 4) + align256(tiles * 4));
   {
-    const int warps = 8;
-    dim3 grid((unsigned)((T + warps - 1) / warps)), block(32 * warps);
-    KernelScope ks("topk_sigmoid", c.stream);
-    const int vpl = (E + 31) / 32;
-    if (vpl <= 1) topk_sigmoid_kernel<1><<<grid, block, 0, c.stream>>>(logits, bias, T, E, K, idx, prob, rowsum);
-    else if (vpl <= 2) topk_sigmoid_kernel<2><<<grid, block, 0, c.stream>>>(logits, bias, T, E, K, idx, prob, rowsum);
-    else if (vpl <= 4) topk_sigmoid_kernel<4><<<grid, block, 0, c.stream>>>(logits, bias, T, E, K, idx, prob, rowsum);
-    else topk_sigmoid_kernel<8><<<grid, block, 0, c.stream>>>(logits, bias, T, E, K, idx, prob, rowsum);
+    const size_t smem = (size_t)(tpb * E + E + tpb + E) * 4;
+    dim3 grid((unsigned)nch, (unsigned)GBS);
+    KernelScope ks("select_sigmoid", c.stream);
+#define MOE_SELECT_SIGMOID(KM)                                                                             \
+  select_sigmoid_kernel<KM><<<grid, 4 * tpb, smem, c.stream>>>(logits, bias, S, E, K, tpb, (int)nch, idx, \
+                                                               prob, psum, pcnt, ticket)
+    switch (sel::k_bound(K)) {
+      case 2: MOE_SELECT_SIGMOID(2); break;
+      case 4: MOE_SELECT_SIGMOID(4); break;
+      case 8: MOE_SELECT_SIGMOID(8); break;
+      default: MOE_SELECT_SIGMOID(16); break;
+    }
+#undef MOE_SELECT_SIGMOID
   }
   cudaError_t st = cudaGetLastError();
   if (st != cudaSuccess) return st;
   {
-    KernelScope ks("aux_partial", c.stream);
-    aux_partial_kernel<<<dim3((unsigned)nchunk, (unsigned)GBS), 256, 0, c.stream>>>(logits, rowsum, idx, S, E, K,
-                                                                                  (int)nchunk, psum, pcnt);
-  }
-  st = cudaGetLastError();
-  if (st != cudaSuccess) return st;
-  {
-    KernelScope ks("aux_finalize", c.stream);
-    aux_finalize_kernel<<<1, 256, 0, c.stream>>>(psum, pcnt, (int)GBS, S, E, K, (int)nchunk, coef, f_out, loss);
+    KernelScope ks("balance_finalize", c.stream);
+    dim3 grid((unsigned)((E + 31) / 32), (unsigned)GBS);
+    balance_finalize_kernel<<<grid, 256, 0, c.stream>>>(psum, pcnt, S, E, K, (int)nch, coef, (int)GBS, f_out,
+                                                        tile_sum, ticket, loss);
   }
   return cudaGetLastError();
 }
@@ -258,9 +283,17 @@ cudaError_t launch_route_dz_sigmoid(const Ctx& c, const float* logits, const int
   const int warps = 8;
   dim3 grid((unsigned)((T + warps - 1) / warps)), block(32 * warps);
   const float cscale = aux_grad * coef / ((float)GBS * (float)S);
+  bf16* d16 = static_cast<bf16*>(dz16);
   KernelScope ks("route_dz_sigmoid", c.stream);
-  route_dz_sigmoid_kernel<<<grid, block, 0, c.stream>>>(logits, idx, prob, dprob, f, T, S, E, K, cscale, dz,
-                                                        static_cast<bf16*>(dz16), c.err);
+#define MOE_DZ_SIGMOID(VPL)                                                                                     \
+  route_dz_sigmoid_kernel<VPL><<<grid, block, 0, c.stream>>>(logits, idx, prob, dprob, f, T, S, E, K, cscale, dz, \
+                                                             d16, c.err)
+  const int vpl = (E + 31) / 32;
+  if (vpl <= 1) MOE_DZ_SIGMOID(1);
+  else if (vpl <= 2) MOE_DZ_SIGMOID(2);
+  else if (vpl <= 4) MOE_DZ_SIGMOID(4);
+  else MOE_DZ_SIGMOID(8);
+#undef MOE_DZ_SIGMOID
   return cudaGetLastError();
 }
 
