@@ -8,3 +8,4 @@ or executes anything here, and this package imports nothing from the product.
 from .moe import *  # noqa: F401,F403
 from .eq1 import *  # noqa: F401,F403
 from .router_sigmoid import *  # noqa: F401,F403
+from .shared import *  # noqa: F401,F403

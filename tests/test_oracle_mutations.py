@@ -145,3 +145,35 @@ def test_sigmoid_router_mistakes_are_caught(monkeypatch):
     monkeypatch.setattr(RS, "seq_aux_loss", wrong_fraction)
     monkeypatch.setattr(oracle, "seq_aux_loss", wrong_fraction)
     _expect_failure(PS.test_balanced_routing_with_flat_scores_gives_the_coefficient)
+
+
+def test_shared_expert_mistakes_are_caught(monkeypatch):
+    import oracle.shared as SE
+    import tests.test_oracle_shared as PSH
+
+    def relu_slope_one(dy, x, h, a, w_s1, w_s2):
+        dA = np.matmul(dy, w_s2)
+        dh = np.maximum(h, 0.0) * dA                   # the factor 2 of d relu^2 dropped
+        return dh, np.matmul(dh, w_s1), np.matmul(dh.T, x), np.matmul(dy.T, a)
+    monkeypatch.setattr(SE, "shared_expert_bwd", relu_slope_one)
+    monkeypatch.setattr(oracle, "shared_expert_bwd", relu_slope_one)
+    _expect_failure(PSH.test_backward_matches_central_differences)
+    monkeypatch.undo()
+
+    def plain_relu(x, w_s1, w_s2):
+        h = np.matmul(x, w_s1.T)
+        a = np.maximum(h, 0.0)                         # square dropped
+        return h, a, np.matmul(a, w_s2.T)
+    monkeypatch.setattr(SE, "shared_expert", plain_relu)
+    monkeypatch.setattr(oracle, "shared_expert", plain_relu)
+    _expect_failure(PSH.test_degree_two_homogeneity_and_sign_gate)
+    monkeypatch.undo()
+
+    def transposed_down(x, w_s1, w_s2):
+        h = np.matmul(x, w_s1.T)
+        a = O_relu_sq(h)
+        return h, a, np.matmul(a, w_s2[:, ::-1].T)      # hidden units matched to the wrong columns
+    O_relu_sq = SE.relu_sq
+    monkeypatch.setattr(SE, "shared_expert", transposed_down)
+    monkeypatch.setattr(oracle, "shared_expert", transposed_down)
+    _expect_failure(PSH.test_forward_is_a_sum_of_squared_positive_projections)
