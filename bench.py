@@ -45,7 +45,7 @@ def _peaks() -> dict:
 # once and each result written once.
 # ---------------------------------------------------------------------------
 
-def kernel_work(name: str, w: synth.Workload, T: int) -> tuple[str, float]:
+def kernel_work(name: str, w: synth.Workload, T: int, Fs: int = 0) -> tuple[str, float]:
     TK, D, E, K, F, bx = T * w.K, w.D, w.E, w.K, w.F, w.b_x
     Din = w.H if w.H else D
     base = name.rsplit("_", 1)[0] if name.endswith(("_tc", "_simt")) else name
@@ -54,6 +54,9 @@ def kernel_work(name: str, w: synth.Workload, T: int) -> tuple[str, float]:
         "ffn2_wgrad": 2.0 * TK * D * F, "ffn1_dgrad": 4.0 * TK * F * D, "ffn1_wgrad": 4.0 * TK * F * D,
         "latent_fwd": 2.0 * T * w.H * D, "latent_dgrad": 2.0 * T * w.H * D, "latent_wgrad": 2.0 * T * w.H * D,
         "router_dgrad": 2.0 * T * Din * E, "router_wgrad": 2.0 * T * Din * E,
+        "shared_fc1": 2.0 * T * Din * Fs, "shared_fc2": 2.0 * T * Fs * Din,
+        "shared_fc2_dgrad": 2.0 * T * Din * Fs, "shared_fc1_dgrad": 2.0 * T * Fs * Din,
+        "shared_fc2_wgrad": 2.0 * T * Din * Fs, "shared_fc1_wgrad": 2.0 * T * Fs * Din,
     }
     if base in flops:
         return "tensor", flops[base]
@@ -70,6 +73,7 @@ def kernel_work(name: str, w: synth.Workload, T: int) -> tuple[str, float]:
         "balance_finalize": 0.0,
         "route_dz_sigmoid": T * E * 4 + T * K * 12 + T * E * 6,
         "swiglu_bwd": 5.0 * TK * F * bx,
+        "relusq_bwd": 3.0 * T * Fs * bx,
         "pack_w1": 0.0,
     }
     return "hbm", float(byts.get(base, 0.0))
@@ -257,6 +261,8 @@ def main() -> None:
     ap.add_argument("--cpu-budget", type=float, default=15.0, help="seconds of CPU work for cpu_baseline")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=10)
+    ap.add_argument("--shared-width", type=int, default=0,
+                    help="hidden units of the ungated shared expert (0 = none; Sec. 5.2)")
     ap.add_argument("--router", default="softmax", choices=["softmax", "sigmoid"],
                     help="softmax top-K, or sigmoid scores + expert bias + sequence-level balance loss (Sec. 5.2)")
     args = ap.parse_args()
@@ -286,7 +292,9 @@ def main() -> None:
     inputs = synth.make_inputs(w, seed=rank_seed(w, rank))      # each rank its own tokens
     if args.router == "sigmoid":
         inputs["expert_bias"] = synth.make_expert_bias(w.E, rank_seed(w, rank))
-    L = MoeLayer(w.S, w.GBS, w.K, w.D, w.E, w.F, w.dtype, w.H, router=args.router)
+    if args.shared_width:
+        inputs.update(synth.make_shared_expert(w, args.shared_width, rank_seed(w, rank)))
+    L = MoeLayer(w.S, w.GBS, w.K, w.D, w.E, w.F, w.dtype, w.H, router=args.router, shared_F=args.shared_width)
     L.load(inputs)
     stream = torch.cuda.current_stream()
     flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device="cuda")
@@ -364,7 +372,7 @@ def main() -> None:
     peaks = _peaks()
     kernels = {}
     for name, (n, ms) in prof.items():
-        bound, work = kernel_work(name, w, T)
+        bound, work = kernel_work(name, w, T, args.shared_width)
         per_launch_ms = ms / max(n, 1)
         kernels[name] = {"launches_per_step": n / args.steps, "ms_per_step": ms / args.steps,
                          "bound": bound, "work_per_launch": work, "avg_launch_ms": per_launch_ms}
@@ -403,7 +411,7 @@ def main() -> None:
               for k, v in sorted(kernels.items(), key=lambda kv: -kv[1]["ms_per_step"])}
 
     cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline and args.router == "softmax":
+    if rank == 0 and world == 1 and not args.no_cpu_baseline and args.router == "softmax" and not args.shared_width:
         cpu = cpu_baseline(w, args.cpu_budget)
 
     if rank == 0:
@@ -412,7 +420,7 @@ def main() -> None:
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": t_max, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
             "config": {"workload": w.name, "T": T, "S": w.S, "GBS": w.GBS, "D": w.D, "E": w.E, "K": w.K, "F": w.F,
-                       "H": w.H, "seed": w.seed, "router": args.router,
+                       "H": w.H, "seed": w.seed, "router": args.router, "shared_width": args.shared_width,
                        "parallelism": f"replicas x{world}, each rank its own tokens",
                        "l2": "256 MiB buffer written before every timed step (outside the step events); "
                              "the step also touches ~3 GB > 129 MB L2"},

@@ -96,7 +96,7 @@ int moe_workspace_size(const moe_shape_t* shape, size_t* bytes);
 int moe_route(const moe_shape_t* shape, const void* x, const void* w_router, const float* bias,
               float* logits, int32_t* topk_idx, float* topk_prob, void* ws, size_t ws_bytes, void* stream);
 
-/* Top-K of given fp32 logits [T, E], one warp per token: the K largest
+/* Top-K of given fp32 logits [T, E] (four threads per token): the K largest
  * logits (ties to the lower expert index), ordered by descending logit, and
  * renormalised probabilities p_k = exp(z_k - z_max) / sum over the K chosen
  * (equal to softmax over all E restricted to the chosen set). */
@@ -217,6 +217,25 @@ int moe_route_sigmoid_bwd(const moe_shape_t* shape, const void* x, const void* w
                           const int32_t* topk_idx, const float* topk_prob, const float* dtopk_prob,
                           const float* aux_f, float aux_coef, float aux_grad, void* dx, float* dw_router,
                           float* dlogits, void* ws, size_t ws_bytes, void* stream);
+
+/* Shared expert (Sec. 5.2 experimental details: an ungated shared expert MLP
+ * in parallel with the routed experts, its output added to the combined routed
+ * output; readings SH1-SH2): with F_s hidden units (a multiple of 64),
+ *   h_save[T, F_s] = x[T, Din] . w_s1^T   (w_s1 [F_s, Din]),
+ *   act_save[T, F_s] = max(h, 0)^2        (squared ReLU, no gate, no biases),
+ *   y[T, Din] += act . w_s2^T             (w_s2 [Din, F_s]; added to the existing
+ *                                          contents, i.e. the routed output).
+ * Call it after the routed output is in y (after the LatentMoE up-projection). */
+int moe_shared_expert(const moe_shape_t* shape, int32_t F_s, const void* x, const void* w_s1, const void* w_s2,
+                      void* h_save, void* act_save, void* y, void* stream);
+
+/* Shared expert backward from dy [T, Din] and the saved h and act:
+ *   dh[T, F_s] = 2 max(h, 0) (dy . w_s2)   (caller's buffer, overwritten),
+ *   dx[T, Din] += dh . w_s1                 (added to the existing contents),
+ *   dw_s1 [F_s, Din] = dh^T . x, dw_s2 [Din, F_s] = dy^T . act (fp32, overwritten). */
+int moe_shared_expert_bwd(const moe_shape_t* shape, int32_t F_s, const void* dy, const void* x, const void* h_save,
+                          const void* act_save, const void* w_s1, const void* w_s2, void* dh, void* dx,
+                          float* dw_s1, float* dw_s2, void* stream);
 
 /* LatentMoE projection (dense, T rows): out[T, n_out] = in[T, n_in] . w^T with
  * w [n_out, n_in].  Down-projection: n_in = H, n_out = D; up-projection:

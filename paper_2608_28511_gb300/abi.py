@@ -33,6 +33,7 @@ EXPORTS = (
     "moe_device_status_word", "moe_last_cuda_error", "moe_strerror", "moe_version", "moe_prof_enable",
     "moe_prof_reset", "moe_prof_count", "moe_prof_get", "moe_launch_count", "moe_dispatch_noalloc",
     "moe_ce_composition", "moe_ce_layer_pattern", "moe_route_sigmoid", "moe_route_sigmoid_bwd",
+    "moe_shared_expert", "moe_shared_expert_bwd",
 )
 
 
@@ -86,6 +87,8 @@ _SIGS = {
     "moe_route_sigmoid": ([_SHP, _VP, _VP, _VP, _F32, _VP, _VP, _VP, _VP, _VP, _VP, _SZ, _VP], ctypes.c_int),
     "moe_route_sigmoid_bwd": ([_SHP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _F32, _F32, _VP, _VP, _VP, _VP, _SZ, _VP],
                               ctypes.c_int),
+    "moe_shared_expert": ([_SHP, _I32, _VP, _VP, _VP, _VP, _VP, _VP, _VP], ctypes.c_int),
+    "moe_shared_expert_bwd": ([_SHP, _I32] + [_VP] * 11, ctypes.c_int),
     "moe_latent_proj": ([_SHP, _I32, _I32, _VP, _VP, _VP, _VP, _SZ, _VP], ctypes.c_int),
     "moe_latent_proj_bwd": ([_SHP, _I32, _I32, _VP, _VP, _VP, _VP, _I32, _VP, _VP, _SZ, _VP], ctypes.c_int),
     "moe_pack_w1": ([_SHP, _VP, _VP, _VP, _VP], ctypes.c_int),
@@ -244,6 +247,17 @@ def moe_route_sigmoid_bwd(shape, x, w_router, logits, topk_idx, topk_prob, dtopk
         _shape(shape), _p(x), _p(w_router), _p(logits), _p(topk_idx), _p(topk_prob), _p(dtopk_prob), _p(aux_f),
         float(aux_coef), float(aux_grad), _p(dx), _p(dw_router), _p(dlogits), _p(ws), _nbytes(ws),
         _stream(stream)))
+
+
+def moe_shared_expert(shape, F_s, x, w_s1, w_s2, h_save, act_save, y, stream=None):
+    _check("moe_shared_expert", lib().moe_shared_expert(_shape(shape), int(F_s), _p(x), _p(w_s1), _p(w_s2),
+                                                        _p(h_save), _p(act_save), _p(y), _stream(stream)))
+
+
+def moe_shared_expert_bwd(shape, F_s, dy, x, h_save, act_save, w_s1, w_s2, dh, dx, dw_s1, dw_s2, stream=None):
+    _check("moe_shared_expert_bwd", lib().moe_shared_expert_bwd(
+        _shape(shape), int(F_s), _p(dy), _p(x), _p(h_save), _p(act_save), _p(w_s1), _p(w_s2), _p(dh), _p(dx),
+        _p(dw_s1), _p(dw_s2), _stream(stream)))
 
 
 def moe_latent_proj(shape, n_in, n_out, x, w, out, ws, stream=None):

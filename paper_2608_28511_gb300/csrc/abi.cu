@@ -864,6 +864,91 @@ int moe_latent_proj_bwd(const moe_shape_t* shape, int32_t n_in, int32_t n_out, c
   return MOE_OK;
 }
 
+// A dense C(m, n) = sum_k A(m, k) B(n, k) descriptor (element strides).
+static GemmDesc dense_desc(Epi epi, int64_t M, int64_t N, int64_t K, const void* A, DType at, int64_t sa_m,
+                           int64_t sa_k, const void* B, DType bt, int64_t sb_n, int64_t sb_k, void* C, DType ct,
+                           int64_t ldc) {
+  GemmDesc g;
+  g.group = Group::Dense;
+  g.epi = epi;
+  g.M = M;
+  g.N = N;
+  g.K = K;
+  g.A = A;
+  g.a_type = at;
+  g.sa_m = sa_m;
+  g.sa_k = sa_k;
+  g.B = B;
+  g.b_type = bt;
+  g.sb_n = sb_n;
+  g.sb_k = sb_k;
+  g.C = C;
+  g.c_type = ct;
+  g.ldc = ldc;
+  return g;
+}
+
+int moe_shared_expert(const moe_shape_t* shape, int32_t F_s, const void* x, const void* w_s1, const void* w_s2,
+                      void* h_save, void* act_save, void* y, void* stream) {
+  Dims d;
+  TRY(check_shape(shape, &d));
+  if (F_s <= 0 || F_s % 64) return MOE_ERR_SHAPE;
+  REQUIRE_PTR(x);
+  REQUIRE_PTR(w_s1);
+  REQUIRE_PTR(w_s2);
+  REQUIRE_PTR(h_save);
+  REQUIRE_PTR(act_save);
+  REQUIRE_PTR(y);
+  Ctx c;
+  TRY(get_ctx(stream, &c));
+  // h = x . w_s1^T, a = relu(h)^2   (M = T, N = F_s, K = Din)
+  GemmDesc g1 = dense_desc(Epi::ReluSqFwd, d.T, F_s, d.Din, x, d.dt, d.Din, 1, w_s1, d.dt, d.Din, 1, h_save, d.dt,
+                           F_s);
+  g1.aux = act_save;
+  TRY_CUDA(gemm(c, g1, "shared_fc1_tc", "shared_fc1_simt"));
+  // y += a . w_s2^T   (M = T, N = Din, K = F_s)
+  GemmDesc g2 = dense_desc(Epi::Accum, d.T, d.Din, F_s, act_save, d.dt, F_s, 1, w_s2, d.dt, F_s, 1, y, d.dt, d.Din);
+  TRY_CUDA(gemm(c, g2, "shared_fc2_tc", "shared_fc2_simt"));
+  return MOE_OK;
+}
+
+int moe_shared_expert_bwd(const moe_shape_t* shape, int32_t F_s, const void* dy, const void* x, const void* h_save,
+                          const void* act_save, const void* w_s1, const void* w_s2, void* dh, void* dx, float* dw_s1,
+                          float* dw_s2, void* stream) {
+  Dims d;
+  TRY(check_shape(shape, &d));
+  if (F_s <= 0 || F_s % 64) return MOE_ERR_SHAPE;
+  REQUIRE_PTR(dy);
+  REQUIRE_PTR(x);
+  REQUIRE_PTR(h_save);
+  REQUIRE_PTR(act_save);
+  REQUIRE_PTR(w_s1);
+  REQUIRE_PTR(w_s2);
+  REQUIRE_PTR(dh);
+  REQUIRE_PTR(dx);
+  REQUIRE_PTR(dw_s1);
+  REQUIRE_PTR(dw_s2);
+  Ctx c;
+  TRY(get_ctx(stream, &c));
+  // dA = dy . w_s2   (M = T, N = F_s, K = Din), into dh
+  GemmDesc a = dense_desc(Epi::Store, d.T, F_s, d.Din, dy, d.dt, d.Din, 1, w_s2, d.dt, 1, F_s, dh, d.dt, F_s);
+  TRY_CUDA(gemm(c, a, "shared_fc2_dgrad_tc", "shared_fc2_dgrad_simt"));
+  // dh = 2 relu(h) dA, in place
+  TRY_CUDA(launch_relusq_bwd(c, d.dt, dh, h_save, d.T * (int64_t)F_s, dh));
+  // dx += dh . w_s1   (M = T, N = Din, K = F_s)
+  GemmDesc b = dense_desc(Epi::Accum, d.T, d.Din, F_s, dh, d.dt, F_s, 1, w_s1, d.dt, 1, d.Din, dx, d.dt, d.Din);
+  TRY_CUDA(gemm(c, b, "shared_fc1_dgrad_tc", "shared_fc1_dgrad_simt"));
+  // dw_s2 = dy^T . a   (M = Din, N = F_s, K = T)
+  GemmDesc w2 = dense_desc(Epi::Store, d.Din, F_s, d.T, dy, d.dt, 1, d.Din, act_save, d.dt, 1, F_s, dw_s2,
+                           DType::F32, F_s);
+  TRY_CUDA(gemm(c, w2, "shared_fc2_wgrad_tc", "shared_fc2_wgrad_simt"));
+  // dw_s1 = dh^T . x   (M = F_s, N = Din, K = T)
+  GemmDesc w1 = dense_desc(Epi::Store, F_s, d.Din, d.T, dh, d.dt, 1, F_s, x, d.dt, 1, d.Din, dw_s1, DType::F32,
+                           d.Din);
+  TRY_CUDA(gemm(c, w1, "shared_fc1_wgrad_tc", "shared_fc1_wgrad_simt"));
+  return MOE_OK;
+}
+
 int moe_pack_w1(const moe_shape_t* shape, const void* w_gate, const void* w_up, void* w1, void* stream) {
   Dims d;
   TRY(check_shape(shape, &d));

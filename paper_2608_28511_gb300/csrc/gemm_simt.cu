@@ -137,6 +137,12 @@ __global__ void __launch_bounds__(256) simt_gemm_kernel(GemmDesc d) {
           }
           break;
         }
+        case Epi::ReluSqFwd: {
+          crow[gn] = from_f32<TC>(v);
+          const float r = fmaxf(v, 0.f);
+          static_cast<TC*>(d.aux)[gm * d.ldc + gn] = from_f32<TC>(r * r);
+          break;
+        }
       }
     }
   }

@@ -83,6 +83,9 @@ bool make_plan(const GemmDesc& d, Plan* pl) {
     case Epi::SwigluFwd:
       if (d.c_type != DType::BF16 || d.N % 128 || !d.aux || !al16(d.aux)) return false;
       break;
+    case Epi::ReluSqFwd:
+      if (d.c_type != DType::BF16 || d.N % 64 || !d.aux || !al16(d.aux)) return false;
+      break;
   }
   pl->bn = 256;
   pl->cg = 1;
@@ -175,7 +178,7 @@ bool gemm_tc_supports(const GemmDesc& d) {
   if (g == 1 && !pl.a_mn && pl.b_mn && e == 0 && !f32) return true;
   if (g == 2 && pl.a_mn && pl.b_mn && e == 0 && f32) return true;
   if (g == 0 && !pl.a_mn && !pl.b_mn && e == 1 && f32) return true;
-  if (g == 0 && !pl.a_mn && !pl.b_mn && e == 0 && !f32) return true;
+  if (g == 0 && !pl.a_mn && !pl.b_mn && (e == 0 || e == 2 || e == 4) && !f32) return true;
   if (g == 0 && !pl.a_mn && pl.b_mn && (e == 0 || e == 2) && !f32) return true;
   if (g == 0 && pl.a_mn && pl.b_mn && e == 0 && f32) return true;
   return false;
@@ -240,6 +243,8 @@ cudaError_t launch_gemm_tc(const Ctx& c, const GemmDesc& d, const char* name) {
     if (g == 1 && !pl.b_mn && e == 0) return launch_inst<256, false, false, 1, 0, bf16, 2>(c, p, ub);
     if (g == 1 && pl.b_mn && e == 0) return launch_inst<256, false, true, 1, 0, bf16, 2>(c, p, ub);
     if (g == 0 && !pl.a_mn && !pl.b_mn && e == 0) return launch_inst<256, false, false, 0, 0, bf16, 2>(c, p, ub);
+    if (g == 0 && !pl.a_mn && !pl.b_mn && e == 2) return launch_inst<256, false, false, 0, 2, bf16, 2>(c, p, ub);
+    if (g == 0 && !pl.a_mn && !pl.b_mn && e == 4) return launch_inst<256, false, false, 0, 4, bf16, 2>(c, p, ub);
     if (g == 0 && !pl.a_mn && pl.b_mn && e == 0) return launch_inst<256, false, true, 0, 0, bf16, 2>(c, p, ub);
     if (g == 0 && !pl.a_mn && pl.b_mn && e == 2) return launch_inst<256, false, true, 0, 2, bf16, 2>(c, p, ub);
     if (g == 0 && pl.a_mn && pl.b_mn) return launch_inst<256, true, true, 0, 0, float, 2>(c, p, ub);
@@ -252,6 +257,8 @@ cudaError_t launch_gemm_tc(const Ctx& c, const GemmDesc& d, const char* name) {
     return launch_inst<256, false, false, 0, 1, float, 1>(c, p, ub);
   }
   if (g == 0 && !pl.a_mn && !pl.b_mn && e == 0) return launch_inst<256, false, false, 0, 0, bf16, 1>(c, p, ub);
+  if (g == 0 && !pl.a_mn && !pl.b_mn && e == 2) return launch_inst<256, false, false, 0, 2, bf16, 1>(c, p, ub);
+  if (g == 0 && !pl.a_mn && !pl.b_mn && e == 4) return launch_inst<256, false, false, 0, 4, bf16, 1>(c, p, ub);
   if (g == 0 && !pl.a_mn && pl.b_mn && e == 0) return launch_inst<256, false, true, 0, 0, bf16, 1>(c, p, ub);
   if (g == 0 && !pl.a_mn && pl.b_mn && e == 2) return launch_inst<256, false, true, 0, 2, bf16, 1>(c, p, ub);
   if (g == 0 && pl.a_mn && pl.b_mn) return launch_inst<256, true, true, 0, 0, float, 1>(c, p, ub);

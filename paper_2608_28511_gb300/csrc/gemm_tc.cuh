@@ -455,7 +455,7 @@ __device__ __forceinline__ void load_row32(const T* src, float* v) {
   for (int i = 0; i < 32; i += NV) unpack16<T>(*reinterpret_cast<const uint4*>(src + i), v + i);
 }
 
-// EPI: 0 Store, 1 StoreBias, 2 Accum, 3 SwigluFwd (values of moe::Epi).
+// EPI: 0 Store, 1 StoreBias, 2 Accum, 3 SwigluFwd, 4 ReluSqFwd (values of moe::Epi).
 // CG: 1 = one CTA per 128 x BN tile; 2 = a cluster of two CTAs per 256 x BN
 // tile (the even CTA issues the MMAs; both stage their halves and drain
 // their own accumulator rows).
@@ -797,7 +797,12 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
                 if (i < nvalid) v[i] += to_f32<TC>(crow[col0 + i]);
             }
             store_row32<TC>(crow + col0, v, nvalid);
-          } else if (EPI == 0) {
+            if (EPI == 4) {
+#pragma unroll
+              for (int i = 0; i < 32; ++i) v[i] = fmaxf(v[i], 0.f) * fmaxf(v[i], 0.f);
+              store_row32<TC>(static_cast<TC*>(p.aux) + grow * p.ldc + col0, v, nvalid);
+            }
+          } else if (EPI == 0 || EPI == 4) {
 #pragma unroll
             for (int r = 0; r < RPC; ++r) {
 #pragma unroll
@@ -806,6 +811,21 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
               stage_put<RB>(stg, lane, pk);
               __syncwarp();
               stage_store<RB>(stg, lane, c_rows + (col0 + r * CPR) * sizeof(TC), ldc_b, nrows);
+            }
+            if (EPI == 4) {
+              // a = relu(h)^2 at the same positions of aux
+              uint8_t* a_rows = reinterpret_cast<uint8_t*>(static_cast<TC*>(p.aux)) + rbase * ldc_b;
+#pragma unroll
+              for (int i = 0; i < 32; ++i) v[i] = fmaxf(v[i], 0.f) * fmaxf(v[i], 0.f);
+#pragma unroll
+              for (int r = 0; r < RPC; ++r) {
+#pragma unroll
+                for (int i = 0; i < NP; ++i) pk[i] = pack16<TC>(v + r * CPR + i * Vec<TC>::N);
+                __syncwarp();
+                stage_put<RB>(stg, lane, pk);
+                __syncwarp();
+                stage_store<RB>(stg, lane, a_rows + (col0 + r * CPR) * sizeof(TC), ldc_b, nrows);
+              }
             }
           }
         }

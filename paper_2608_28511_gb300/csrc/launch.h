@@ -94,6 +94,8 @@ cudaError_t launch_pack_w1(const Ctx& c, DType dt, const void* w_gate, const voi
 // swiglu.cu: dH [rows, 2F] (packed) from dA [rows, F] and the saved h [rows, 2F].
 cudaError_t launch_swiglu_bwd(const Ctx& c, DType dt, const void* dA, const void* h, int64_t rows, int F,
                               void* dH);
+// swiglu.cu: dh = 2 max(h, 0) dA over n elements (dh may alias dA).
+cudaError_t launch_relusq_bwd(const Ctx& c, DType dt, const void* dA, const void* h, int64_t n, void* dh);
 
 // ---------------------------------------------------------------------------
 // Grouped GEMM  C(m, n) = sum_k A(m, k) B(n, k), fp32 accumulation.
@@ -109,6 +111,7 @@ enum class Epi : int {
   StoreBias = 1,  // C = acc + bias[n]
   Accum = 2,      // C = C + acc
   SwigluFwd = 3,  // acc is h (packed gate/up, N = 2F): C = h, aux[m, f] = silu(g) u  (aux ld = N/2)
+  ReluSqFwd = 4,  // acc is h: C = h, aux[m, n] = max(h, 0)^2  (aux ld = ldc)
 };
 
 struct GemmDesc {
@@ -128,7 +131,7 @@ struct GemmDesc {
   DType c_type = DType::BF16;
   int64_t ldc = 0, sc_g = 0;
   const float* bias = nullptr;       // StoreBias
-  void* aux = nullptr;               // SwigluFwd activation output (c_type)
+  void* aux = nullptr;               // SwigluFwd / ReluSqFwd activation output (c_type)
   void* scratch = nullptr;           // Group::K on the tensor-core engine: per-group tensor maps
                                      // (gemm_tc_group_scratch_bytes, 128-byte aligned)
   int64_t split_rows = 0;            // Group::K with offsets == nullptr: num_groups equal splits of

@@ -24,10 +24,12 @@ class MoeLayer:
     ``router="sigmoid"`` with sigmoid scores, a selection-only expert bias and
     the sequence-level balance loss (coefficient ``aux_coef``; its gradient
     enters the backward pass scaled by ``aux_grad``), Sec. 5.2.
+    ``shared_F > 0`` adds the ungated shared expert of that width (Sec. 5.2),
+    whose output is added to the layer output.
     """
 
     def __init__(self, S, GBS, K, D, E, F, dtype="bf16", H=0, device="cuda", router="softmax", aux_coef=1e-4,
-                 aux_grad=1.0):
+                 aux_grad=1.0, shared_F=0):
         if router not in ("softmax", "sigmoid"):
             raise ValueError(f"unknown router {router!r}")
         self.router = router
@@ -50,6 +52,9 @@ class MoeLayer:
         self.w2 = e(E, D, F)
         self.bias = None
         self.expert_bias = torch.zeros(E, dtype=f32, device=dev) if router == "sigmoid" else None
+        self.shared_F = Fs = int(shared_F)
+        self.w_s1 = e(Fs, self.Din) if Fs else None
+        self.w_s2 = e(self.Din, Fs) if Fs else None
         self.w_down = e(D, H) if H else None
         self.w_upp = e(H, D) if H else None
         # forward
@@ -70,6 +75,11 @@ class MoeLayer:
         self.y_perm = e(TK, D)
         self.y_lat = e(T, D) if H else None
         self.y = e(T, Din)
+        self.h_s = e(T, Fs) if Fs else None
+        self.act_s = e(T, Fs) if Fs else None
+        self.dh_s = e(T, Fs) if Fs else None
+        self.dw_s1 = e(Fs, Din, d=f32) if Fs else None
+        self.dw_s2 = e(Din, Fs, d=f32) if Fs else None
         # backward
         self.dy = e(T, Din)
         self.dy_lat = e(T, D) if H else None
@@ -104,6 +114,9 @@ class MoeLayer:
             self.bias = inputs["bias"].to(self.x.device, non_blocking=True).contiguous()
         else:
             self.bias = None
+        if self.shared_F:
+            self.w_s1.copy_(inputs["w_s1"], non_blocking=True)
+            self.w_s2.copy_(inputs["w_s2"], non_blocking=True)
         if self.router == "sigmoid" and inputs.get("expert_bias") is not None:
             self.expert_bias.copy_(inputs["expert_bias"], non_blocking=True)
 
@@ -129,6 +142,9 @@ class MoeLayer:
             abi.moe_latent_proj(s, self.D, self.H, self.y_lat, self.w_upp, self.y, self.ws, stream)
         else:
             abi.moe_combine(s, self.y_perm, self.prob_perm, self.row_of_slot, self.y, stream)
+        if self.shared_F:
+            abi.moe_shared_expert(s, self.shared_F, self.x, self.w_s1, self.w_s2, self.h_s, self.act_s, self.y,
+                                  stream)
         return self.y
 
     def backward(self, stream=None):
@@ -155,6 +171,9 @@ class MoeLayer:
         else:
             abi.moe_route_bwd(s, self.x, self.w_router, self.topk_idx, self.topk_prob, self.dprob, self.dx,
                               self.dw_router, self.dlogits, self.ws, stream)
+        if self.shared_F:
+            abi.moe_shared_expert_bwd(s, self.shared_F, self.dy, self.x, self.h_s, self.act_s, self.w_s1, self.w_s2,
+                                      self.dh_s, self.dx, self.dw_s1, self.dw_s2, stream)
         return self.dx
 
     def step(self, stream=None):

@@ -27,6 +27,8 @@ Public layouts (row-major):
   bias    [E] float32   per-expert logit bias (skewed workload only)
   expert_bias [E] float32  selection-only bias of the sigmoid router
                         (``make_expert_bias``, drawn separately)
+  w_s1 [F_s, D], w_s2 [D, F_s]  shared expert (``make_shared_expert``, drawn
+                        separately; LatentMoE: H in place of D)
   dy      [T, D]        upstream gradient (LatentMoE: [T, H])
 """
 from __future__ import annotations
@@ -101,6 +103,17 @@ def make_expert_bias(E: int, seed: int, std: float = 0.05) -> torch.Tensor:
     generator (seed + 7919), so it leaves the ``make_inputs`` stream alone."""
     g = torch.Generator().manual_seed(int(seed) + 7919)
     return torch.randn(E, generator=g, dtype=torch.float32) * std
+
+
+def make_shared_expert(w: Workload, F_s: int, seed: int) -> dict:
+    """Shared-expert weights w_s1 [F_s, Din] and w_s2 [Din, F_s] in the storage
+    dtype, N(0, 1/fan_in) from their own generator (seed + 104729)."""
+    g = torch.Generator().manual_seed(int(seed) + 104729)
+    X = w.in_width
+    st = _storage(w.dtype)
+    w1 = (torch.randn(F_s, X, generator=g, dtype=torch.float32) / math.sqrt(X)).to(st)
+    w2 = (torch.randn(X, F_s, generator=g, dtype=torch.float32) / math.sqrt(F_s)).to(st)
+    return {"w_s1": w1, "w_s2": w2}
 
 
 def _storage(dtype: str) -> torch.dtype:
