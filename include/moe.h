@@ -151,6 +151,16 @@ int moe_expert_ffn(const moe_shape_t* shape, const void* x_perm, const int32_t* 
                    const void* w1, const void* w2, void* h_save, void* act_save, void* y_perm,
                    void* ws, size_t ws_bytes, void* stream);
 
+/* moe_expert_ffn with GEMM-1 reading its rows straight from the dispatch
+ * input: row r of expert e is x[token_of_row[r]] (x [T, D]; for LatentMoE the
+ * down-projected x_lat), loaded by the copy engine's four-row gathers, so the
+ * dispatched copy x_perm is never written (moe_dispatch may then be called
+ * with x_perm = NULL).  Same results as moe_expert_ffn on
+ * x_perm = x[token_of_row]. */
+int moe_expert_ffn_gather(const moe_shape_t* shape, const void* x, const int32_t* token_of_row,
+                          const int32_t* expert_offsets, const void* w1, const void* w2, void* h_save,
+                          void* act_save, void* y_perm, void* ws, size_t ws_bytes, void* stream);
+
 /* Combine (forward hidden combine, Sec. 4.1 footnote; reading R5):
  * y[t] = sum_k prob_perm[r] * y_perm[r], r = row_of_slot[t K + k], fp32
  * accumulation, one rounding to the storage dtype.  y is [T, D]. */
@@ -170,6 +180,13 @@ int moe_combine_bwd(const moe_shape_t* shape, const void* dy, const void* y_perm
 int moe_expert_ffn_bwd(const moe_shape_t* shape, const void* dy_perm, const void* x_perm, const void* h_save,
                        const void* act_save, const int32_t* expert_offsets, const void* w1, const void* w2,
                        void* dx_perm, float* dw1, float* dw2, void* ws, size_t ws_bytes, void* stream);
+
+/* moe_expert_ffn_bwd whose GEMM-1 weight gradient gathers the rows of x
+ * [T, D] by token_of_row instead of reading x_perm (same results). */
+int moe_expert_ffn_bwd_gather(const moe_shape_t* shape, const void* dy_perm, const void* x,
+                              const int32_t* token_of_row, const void* h_save, const void* act_save,
+                              const int32_t* expert_offsets, const void* w1, const void* w2, void* dx_perm,
+                              float* dw1, float* dw2, void* ws, size_t ws_bytes, void* stream);
 
 /* Dispatch backward (inverse of the hidden and probability dispatches):
  * dx[t] = sum_k dx_perm[r] (fp32 accumulation; dx [T, D] is overwritten) and

@@ -33,7 +33,7 @@ EXPORTS = (
     "moe_device_status_word", "moe_last_cuda_error", "moe_strerror", "moe_version", "moe_prof_enable",
     "moe_prof_reset", "moe_prof_count", "moe_prof_get", "moe_launch_count", "moe_dispatch_noalloc",
     "moe_ce_composition", "moe_ce_layer_pattern", "moe_route_sigmoid", "moe_route_sigmoid_bwd",
-    "moe_shared_expert", "moe_shared_expert_bwd",
+    "moe_shared_expert", "moe_shared_expert_bwd", "moe_expert_ffn_gather", "moe_expert_ffn_bwd_gather",
 )
 
 
@@ -87,6 +87,8 @@ _SIGS = {
     "moe_route_sigmoid": ([_SHP, _VP, _VP, _VP, _F32, _VP, _VP, _VP, _VP, _VP, _VP, _SZ, _VP], ctypes.c_int),
     "moe_route_sigmoid_bwd": ([_SHP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _F32, _F32, _VP, _VP, _VP, _VP, _SZ, _VP],
                               ctypes.c_int),
+    "moe_expert_ffn_gather": ([_SHP] + [_VP] * 9 + [_SZ, _VP], ctypes.c_int),
+    "moe_expert_ffn_bwd_gather": ([_SHP] + [_VP] * 12 + [_SZ, _VP], ctypes.c_int),
     "moe_shared_expert": ([_SHP, _I32, _VP, _VP, _VP, _VP, _VP, _VP, _VP], ctypes.c_int),
     "moe_shared_expert_bwd": ([_SHP, _I32] + [_VP] * 11, ctypes.c_int),
     "moe_latent_proj": ([_SHP, _I32, _I32, _VP, _VP, _VP, _VP, _SZ, _VP], ctypes.c_int),
@@ -204,6 +206,20 @@ def moe_expert_ffn(shape, x_perm, expert_offsets, w1, w2, h_save, act_save, y_pe
     _check("moe_expert_ffn", lib().moe_expert_ffn(_shape(shape), _p(x_perm), _p(expert_offsets), _p(w1), _p(w2),
                                                   _p(h_save), _p(act_save), _p(y_perm), _p(ws), _nbytes(ws),
                                                   _stream(stream)))
+
+
+def moe_expert_ffn_gather(shape, x, token_of_row, expert_offsets, w1, w2, h_save, act_save, y_perm, ws,
+                          stream=None):
+    _check("moe_expert_ffn_gather", lib().moe_expert_ffn_gather(
+        _shape(shape), _p(x), _p(token_of_row), _p(expert_offsets), _p(w1), _p(w2), _p(h_save), _p(act_save),
+        _p(y_perm), _p(ws), _nbytes(ws), _stream(stream)))
+
+
+def moe_expert_ffn_bwd_gather(shape, dy_perm, x, token_of_row, h_save, act_save, expert_offsets, w1, w2, dx_perm,
+                              dw1, dw2, ws, stream=None):
+    _check("moe_expert_ffn_bwd_gather", lib().moe_expert_ffn_bwd_gather(
+        _shape(shape), _p(dy_perm), _p(x), _p(token_of_row), _p(h_save), _p(act_save), _p(expert_offsets), _p(w1),
+        _p(w2), _p(dx_perm), _p(dw1), _p(dw2), _p(ws), _nbytes(ws), _stream(stream)))
 
 
 def moe_combine(shape, y_perm, prob_perm, row_of_slot, y, stream=None):

@@ -378,22 +378,12 @@ int moe_dispatch(const moe_shape_t* shape, const void* x, const int32_t* topk_id
   return MOE_OK;
 }
 
-int moe_expert_ffn(const moe_shape_t* shape, const void* x_perm, const int32_t* expert_offsets, const void* w1,
-                   const void* w2, void* h_save, void* act_save, void* y_perm, void* ws, size_t ws_bytes,
-                   void* stream) {
-  Dims d;
-  TRY(check_shape(shape, &d));
-  REQUIRE_PTR(x_perm);
-  REQUIRE_PTR(expert_offsets);
-  REQUIRE_PTR(w1);
-  REQUIRE_PTR(w2);
-  REQUIRE_PTR(h_save);
-  REQUIRE_PTR(act_save);
-  REQUIRE_PTR(y_perm);
-  (void)ws;
-  (void)ws_bytes;
-  Ctx c;
-  TRY(get_ctx(stream, &c));
+// The expert FFN with GEMM-1's A rows either read in order (x_rows = x_perm,
+// gather = NULL) or gathered from the dispatch input (x_rows = x [T, D],
+// gather = token_of_row).
+static int expert_ffn_impl(const Ctx& c, const Dims& d, const void* x_rows, const int32_t* gather,
+                           const int32_t* expert_offsets, const void* w1, const void* w2, void* h_save,
+                           void* act_save, void* y_perm) {
   if (d.TK == 0) return MOE_OK;
   // GEMM-1 + fused SwiGLU: h = x_perm . w1_e^T, a = silu(g) * u
   GemmDesc g1;
@@ -404,10 +394,12 @@ int moe_expert_ffn(const moe_shape_t* shape, const void* x_perm, const int32_t* 
   g1.num_groups = d.E;
   g1.offsets = expert_offsets;
   g1.max_rows = d.TK;
-  g1.A = x_perm;
+  g1.A = x_rows;
   g1.a_type = d.dt;
   g1.sa_m = d.D;
   g1.sa_k = 1;
+  g1.gather = gather;
+  g1.gather_rows = d.T;
   g1.B = w1;
   g1.b_type = d.dt;
   g1.sb_n = d.D;
@@ -443,6 +435,45 @@ int moe_expert_ffn(const moe_shape_t* shape, const void* x_perm, const int32_t* 
   return MOE_OK;
 }
 
+int moe_expert_ffn(const moe_shape_t* shape, const void* x_perm, const int32_t* expert_offsets, const void* w1,
+                   const void* w2, void* h_save, void* act_save, void* y_perm, void* ws, size_t ws_bytes,
+                   void* stream) {
+  Dims d;
+  TRY(check_shape(shape, &d));
+  REQUIRE_PTR(x_perm);
+  REQUIRE_PTR(expert_offsets);
+  REQUIRE_PTR(w1);
+  REQUIRE_PTR(w2);
+  REQUIRE_PTR(h_save);
+  REQUIRE_PTR(act_save);
+  REQUIRE_PTR(y_perm);
+  (void)ws;
+  (void)ws_bytes;
+  Ctx c;
+  TRY(get_ctx(stream, &c));
+  return expert_ffn_impl(c, d, x_perm, nullptr, expert_offsets, w1, w2, h_save, act_save, y_perm);
+}
+
+int moe_expert_ffn_gather(const moe_shape_t* shape, const void* x, const int32_t* token_of_row,
+                          const int32_t* expert_offsets, const void* w1, const void* w2, void* h_save,
+                          void* act_save, void* y_perm, void* ws, size_t ws_bytes, void* stream) {
+  Dims d;
+  TRY(check_shape(shape, &d));
+  REQUIRE_PTR(x);
+  REQUIRE_PTR(token_of_row);
+  REQUIRE_PTR(expert_offsets);
+  REQUIRE_PTR(w1);
+  REQUIRE_PTR(w2);
+  REQUIRE_PTR(h_save);
+  REQUIRE_PTR(act_save);
+  REQUIRE_PTR(y_perm);
+  (void)ws;
+  (void)ws_bytes;
+  Ctx c;
+  TRY(get_ctx(stream, &c));
+  return expert_ffn_impl(c, d, x, token_of_row, expert_offsets, w1, w2, h_save, act_save, y_perm);
+}
+
 int moe_combine(const moe_shape_t* shape, const void* y_perm, const float* prob_perm, const int32_t* row_of_slot,
                 void* y, void* stream) {
   Dims d;
@@ -473,25 +504,12 @@ int moe_combine_bwd(const moe_shape_t* shape, const void* dy, const void* y_perm
   return MOE_OK;
 }
 
-int moe_expert_ffn_bwd(const moe_shape_t* shape, const void* dy_perm, const void* x_perm, const void* h_save,
-                       const void* act_save, const int32_t* expert_offsets, const void* w1, const void* w2,
-                       void* dx_perm, float* dw1, float* dw2, void* ws, size_t ws_bytes, void* stream) {
-  Dims d;
-  TRY(check_shape(shape, &d));
-  REQUIRE_PTR(dy_perm);
-  REQUIRE_PTR(x_perm);
-  REQUIRE_PTR(h_save);
-  REQUIRE_PTR(act_save);
-  REQUIRE_PTR(expert_offsets);
-  REQUIRE_PTR(w1);
-  REQUIRE_PTR(w2);
-  REQUIRE_PTR(dx_perm);
-  REQUIRE_PTR(dw1);
-  REQUIRE_PTR(dw2);
-  REQUIRE_PTR(ws);
-  if (ws_bytes < ws_ffn_bwd(d)) return MOE_ERR_WORKSPACE;
-  Ctx c;
-  TRY(get_ctx(stream, &c));
+// Expert FFN backward; the weight gradient of GEMM-1 reads x_rows in order
+// (x_perm, gather = NULL) or gathers them from x [T, D] by token_of_row.
+static int expert_ffn_bwd_impl(const Ctx& c, const Dims& d, const void* dy_perm, const void* x_rows,
+                               const int32_t* gather, const void* h_save, const void* act_save,
+                               const int32_t* expert_offsets, const void* w1, const void* w2, void* dx_perm,
+                               float* dw1, float* dw2, void* ws) {
   void* dH = ws;
   void* dA = static_cast<char*>(ws) + (size_t)d.TK * 2 * d.F * d.bx;
   void* maps = static_cast<char*>(ws) + ws_ffn_bwd_maps_offset(d);
@@ -571,10 +589,12 @@ int moe_expert_ffn_bwd(const moe_shape_t* shape, const void* dy_perm, const void
   w.a_type = d.dt;
   w.sa_m = 1;
   w.sa_k = 2 * d.F;
-  w.B = x_perm;
+  w.B = x_rows;
   w.b_type = d.dt;
   w.sb_n = 1;
   w.sb_k = d.D;
+  w.gather = gather;
+  w.gather_rows = d.T;
   w.max_rows = d.TK;
   w.scratch = maps;
   w.C = dw1;
@@ -589,6 +609,54 @@ int moe_expert_ffn_bwd(const moe_shape_t* shape, const void* dy_perm, const void
   if (d.TK > 0) TRY_CUDA(gemm(c, cg, "ffn1_dgrad_tc", "ffn1_dgrad_simt"));
   TRY_CUDA(gemm(c, w, "ffn1_wgrad_tc", "ffn1_wgrad_simt"));
   return MOE_OK;
+}
+
+int moe_expert_ffn_bwd(const moe_shape_t* shape, const void* dy_perm, const void* x_perm, const void* h_save,
+                       const void* act_save, const int32_t* expert_offsets, const void* w1, const void* w2,
+                       void* dx_perm, float* dw1, float* dw2, void* ws, size_t ws_bytes, void* stream) {
+  Dims d;
+  TRY(check_shape(shape, &d));
+  REQUIRE_PTR(dy_perm);
+  REQUIRE_PTR(x_perm);
+  REQUIRE_PTR(h_save);
+  REQUIRE_PTR(act_save);
+  REQUIRE_PTR(expert_offsets);
+  REQUIRE_PTR(w1);
+  REQUIRE_PTR(w2);
+  REQUIRE_PTR(dx_perm);
+  REQUIRE_PTR(dw1);
+  REQUIRE_PTR(dw2);
+  REQUIRE_PTR(ws);
+  if (ws_bytes < ws_ffn_bwd(d)) return MOE_ERR_WORKSPACE;
+  Ctx c;
+  TRY(get_ctx(stream, &c));
+  return expert_ffn_bwd_impl(c, d, dy_perm, x_perm, nullptr, h_save, act_save, expert_offsets, w1, w2, dx_perm,
+                             dw1, dw2, ws);
+}
+
+int moe_expert_ffn_bwd_gather(const moe_shape_t* shape, const void* dy_perm, const void* x,
+                              const int32_t* token_of_row, const void* h_save, const void* act_save,
+                              const int32_t* expert_offsets, const void* w1, const void* w2, void* dx_perm,
+                              float* dw1, float* dw2, void* ws, size_t ws_bytes, void* stream) {
+  Dims d;
+  TRY(check_shape(shape, &d));
+  REQUIRE_PTR(dy_perm);
+  REQUIRE_PTR(x);
+  REQUIRE_PTR(token_of_row);
+  REQUIRE_PTR(h_save);
+  REQUIRE_PTR(act_save);
+  REQUIRE_PTR(expert_offsets);
+  REQUIRE_PTR(w1);
+  REQUIRE_PTR(w2);
+  REQUIRE_PTR(dx_perm);
+  REQUIRE_PTR(dw1);
+  REQUIRE_PTR(dw2);
+  REQUIRE_PTR(ws);
+  if (ws_bytes < ws_ffn_bwd(d)) return MOE_ERR_WORKSPACE;
+  Ctx c;
+  TRY(get_ctx(stream, &c));
+  return expert_ffn_bwd_impl(c, d, dy_perm, x, token_of_row, h_save, act_save, expert_offsets, w1, w2, dx_perm,
+                             dw1, dw2, ws);
 }
 
 int moe_dispatch_bwd(const moe_shape_t* shape, const void* dx_perm, const float* dprob_perm,

@@ -3,7 +3,7 @@
 //
 // C(m, n) = sum_k A(m, k) B(n, k) with arbitrary element strides, grouped
 // along M (per-expert row ranges), along K (per-expert reduction ranges) or
-// dense, plus the router / SwiGLU epilogues.  Tile 64 x 128 x 16, 256
+// dense, plus the router / SwiGLU epilogues, and the row gathers of GemmDesc.  Tile 64 x 128 x 16, 256
 // threads; thread (ty, tx) owns rows 4 ty .. 4 ty + 3 and columns
 // 4 tx .. 4 tx + 3 and 64 + 4 tx .. 64 + 4 tx + 3 of the tile, so a packed
 // gate column and its up column (64 apart) land in the same thread.
@@ -75,7 +75,10 @@ __global__ void __launch_bounds__(256) simt_gemm_kernel(GemmDesc d) {
       if (a_kfast) { k = i % BK; m = i / BK; } else { m = i % BM; k = i / BM; }
       const int64_t gm = row0 + m, gk = k0 + k;
       float v = 0.f;
-      if (gm < row_end && gk < kend) v = ldf<TA>(d.A, gm * d.sa_m + gk * d.sa_k);
+      if (gm < row_end && gk < kend) {
+        const int64_t sm = (d.gather && d.group == Group::M) ? (int64_t)d.gather[gm] : gm;
+        v = ldf<TA>(d.A, sm * d.sa_m + gk * d.sa_k);
+      }
       As[k][m] = v;
     }
     for (int i = tid; i < BN * BK; i += 256) {
@@ -83,7 +86,10 @@ __global__ void __launch_bounds__(256) simt_gemm_kernel(GemmDesc d) {
       if (b_kfast) { k = i % BK; n = i / BK; } else { n = i % BN; k = i / BN; }
       const int64_t gn = n0 + n, gk = k0 + k;
       float v = 0.f;
-      if (gn < d.N && gk < kend) v = ldf<TB>(Bp, gn * d.sb_n + gk * d.sb_k);
+      if (gn < d.N && gk < kend) {
+        const int64_t sk = (d.gather && d.group == Group::K) ? (int64_t)d.gather[gk] : gk;
+        v = ldf<TB>(Bp, gn * d.sb_n + sk * d.sb_k);
+      }
       Bs[k][n] = v;
     }
     __syncthreads();

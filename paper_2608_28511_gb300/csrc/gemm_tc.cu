@@ -74,6 +74,11 @@ bool make_plan(const GemmDesc& d, Plan* pl) {
   if (d.group == Group::M && (d.sb_g % pl->ldb)) return false;
   if (d.group != Group::Dense && (d.num_groups <= 0 || d.num_groups > kMaxE)) return false;
   if (d.group == Group::M && !d.offsets) return false;
+  if (d.gather) {
+    // gathered operand: K-major A of Group::M or MN-major B of Group::K
+    if (d.gather_rows <= 0 || d.group == Group::Dense) return false;
+    if (d.group == Group::M && pl->a_mn) return false;
+  }
   const size_t cs = dsize(d.c_type);
   if ((d.ldc * cs) % 16) return false;
   switch (d.epi) {
@@ -120,9 +125,9 @@ int max_pair_clusters(KernelT k, int smem, int threads) {
 }
 
 // ub = upper bound on the number of tiles (each tile is one CTA, or one pair for CG 2).
-template <int BN, bool A_MN, bool B_MN, int GROUP, int EPI, typename TC, int CG>
+template <int BN, bool A_MN, bool B_MN, int GROUP, int EPI, typename TC, int CG, int GATHER = 0>
 cudaError_t launch_inst(const Ctx& c, const Params& p, int64_t ub) {
-  auto k = tc::gemm_tc_kernel<BN, A_MN, B_MN, GROUP, EPI, TC, CG>;
+  auto k = tc::gemm_tc_kernel<BN, A_MN, B_MN, GROUP, EPI, TC, CG, GATHER>;
   constexpr int kSmem = Cfg<BN, CG, sizeof(TC)>::kSmem;
   constexpr int kThreads = Cfg<BN, CG, sizeof(TC)>::kThreads;
   static bool configured = false;
@@ -172,6 +177,11 @@ bool gemm_tc_supports(const GemmDesc& d) {
   if (!make_plan(d, &pl)) return false;
   const int g = (int)d.group, e = (int)d.epi;
   const bool f32 = d.c_type == DType::F32;
+  if (d.gather) {
+    if (g == 1 && !pl.b_mn && e == 3 && !f32 && pl.cg == 2) return true;  // GEMM-1 + SwiGLU from x
+    if (g == 2 && e == 0 && f32) return true;                            // GEMM-1 weight gradient from x
+    return false;
+  }
   // the instantiated combinations
   if (g == 1 && !pl.a_mn && !pl.b_mn && e == 3 && !f32) return true;
   if (g == 1 && !pl.a_mn && !pl.b_mn && e == 0 && !f32) return true;
@@ -191,16 +201,22 @@ cudaError_t launch_gemm_tc(const Ctx& c, const GemmDesc& d, const char* name) {
   memset(&p, 0, sizeof(p));
   const int bn = pl.bn, bmp = BM * pl.cg, bnc = bn / pl.cg;
   // A: K-major box {64 k, 128 m}; MN-major box {64 m, 64 k}
-  const int64_t a_rows = pl.a_mn ? (d.group == Group::K ? d.max_rows : d.K) : (d.group == Group::M ? d.max_rows : d.M);
+  const bool ga = d.gather && d.group == Group::M;  // A's rows gathered (one-row box)
+  const bool gb = d.gather && d.group == Group::K;  // B's k rows gathered (one-row box)
+  int64_t a_rows = pl.a_mn ? (d.group == Group::K ? d.max_rows : d.K) : (d.group == Group::M ? d.max_rows : d.M);
+  if (ga) a_rows = d.gather_rows;
   const int64_t a_inner = pl.a_mn ? d.M : d.K;
-  if (!make_map(&p.ta, d.A, a_inner, a_rows, pl.lda * 2, 64, pl.a_mn ? 64 : BM)) return cudaErrorInvalidValue;
+  if (!make_map(&p.ta, d.A, a_inner, a_rows, pl.lda * 2, 64, ga ? 1 : (pl.a_mn ? 64 : BM)))
+    return cudaErrorInvalidValue;
   // B: K-major box {64 k, BN / CG n}; MN-major box {64 n, 64 k}
   const int64_t grows = d.group == Group::M ? d.sb_g / pl.ldb : 0;
   int64_t b_rows;
   if (pl.b_mn) b_rows = d.group == Group::M ? grows * d.num_groups : (d.group == Group::K ? d.max_rows : d.K);
   else b_rows = d.group == Group::M ? grows * d.num_groups : d.N;
+  if (gb) b_rows = d.gather_rows;
   const int64_t b_inner = pl.b_mn ? d.N : d.K;
-  if (!make_map(&p.tb, d.B, b_inner, b_rows, pl.ldb * 2, 64, pl.b_mn ? 64 : bnc)) return cudaErrorInvalidValue;
+  if (!make_map(&p.tb, d.B, b_inner, b_rows, pl.ldb * 2, 64, gb ? 1 : (pl.b_mn ? 64 : bnc)))
+    return cudaErrorInvalidValue;
   p.M = d.M;
   p.N = d.N;
   p.K = d.K;
@@ -215,6 +231,7 @@ cudaError_t launch_gemm_tc(const Ctx& c, const GemmDesc& d, const char* name) {
   p.bias = d.bias;
   p.aux = d.aux;
   p.err = c.err;
+  p.gather = d.gather;
   int64_t ub;
   if (d.group == Group::Dense) ub = (int64_t)p.tiles_m * p.tiles_n;
   else if (d.group == Group::M) ub = ((d.max_rows + bmp - 1) / bmp + d.num_groups) * p.tiles_n;
@@ -229,7 +246,7 @@ cudaError_t launch_gemm_tc(const Ctx& c, const GemmDesc& d, const char* name) {
       KernelScope ks("group_maps", c.stream);
       tc::build_group_maps<<<(d.num_groups + 127) / 128, 128, 0, c.stream>>>(
           p.ta, p.tb, d.offsets, d.num_groups, d.split_rows, split_offs, static_cast<const uint8_t*>(d.A),
-          pl.lda * 2, static_cast<const uint8_t*>(d.B), pl.ldb * 2, maps);
+          pl.lda * 2, gb ? nullptr : static_cast<const uint8_t*>(d.B), pl.ldb * 2, maps);
     }
     cudaError_t st = cudaGetLastError();
     if (st != cudaSuccess) return st;
@@ -237,6 +254,9 @@ cudaError_t launch_gemm_tc(const Ctx& c, const GemmDesc& d, const char* name) {
     if (split_offs) p.offsets = split_offs;
   }
   KernelScope ks(name, c.stream);
+  if (ga) return launch_inst<256, false, false, 1, 3, bf16, 2, 1>(c, p, ub);
+  if (gb && pl.cg == 2) return launch_inst<256, true, true, 2, 0, float, 2, 2>(c, p, ub);
+  if (gb) return launch_inst<256, true, true, 2, 0, float, 1, 2>(c, p, ub);
   if (pl.cg == 2) {
     if (g == 2) return launch_inst<256, true, true, 2, 0, float, 2>(c, p, ub);
     if (g == 1 && !pl.b_mn && e == 3) return launch_inst<256, false, false, 1, 3, bf16, 2>(c, p, ub);

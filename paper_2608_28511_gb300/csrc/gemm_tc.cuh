@@ -47,6 +47,7 @@ struct Params {
   void* aux;
   uint32_t* err;
   const CUtensorMap* gmaps;  // Group::K: per group {A, B} maps whose rows start at the group's first row
+  const int32_t* gather;     // GATHER: source row of each gathered row (the permutation's token_of_row)
 };
 
 // ---------------------------------------------------------------------------
@@ -192,6 +193,24 @@ __device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const CUtensorMap
       "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%3, "
       "%4}], [%2];" ::"r"(dst),
       "l"(reinterpret_cast<uint64_t>(map)), "r"(bar_cluster), "r"(x), "r"(y)
+      : "memory");
+}
+// Four rows r0..r3 of a 2-D tensor map with a one-row box, columns [x, x + box),
+// into 4 consecutive 128-byte rows of shared memory (swizzled like a tiled copy).
+__device__ __forceinline__ void tma_gather4(uint32_t dst, const CUtensorMap* map, uint32_t bar, int x, int r0, int r1,
+                                            int r2, int r3) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile::gather4.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4, "
+      "%5, %6, %7}], [%2];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(x), "r"(r0), "r"(r1), "r"(r2), "r"(r3)
+      : "memory");
+}
+__device__ __forceinline__ void tma_gather4_pair(uint32_t dst, const CUtensorMap* map, uint32_t bar_cluster, int x,
+                                                 int r0, int r1, int r2, int r3) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.tile::gather4.mbarrier::complete_tx::bytes [%0], "
+      "[%1, {%3, %4, %5, %6, %7}], [%2];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar_cluster), "r"(x), "r"(r0), "r"(r1), "r"(r2), "r"(r3)
       : "memory");
 }
 template <int CG>
@@ -459,7 +478,10 @@ __device__ __forceinline__ void load_row32(const T* src, float* v) {
 // CG: 1 = one CTA per 128 x BN tile; 2 = a cluster of two CTAs per 256 x BN
 // tile (the even CTA issues the MMAs; both stage their halves and drain
 // their own accumulator rows).
-template <int BN, bool A_MN, bool B_MN, int GROUP, int EPI, typename TC, int CG>
+// GATHER: 0 tiled copies; 1 A's rows (K-major, Group::M) and 2 B's k rows
+// (MN-major, Group::K) are gathered from a source matrix through p.gather
+// (row -> source row), four rows per copy, by the 32 lanes of the producer warp.
+template <int BN, bool A_MN, bool B_MN, int GROUP, int EPI, typename TC, int CG, int GATHER = 0>
 __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
     gemm_tc_kernel(const __grid_constant__ Params p) {
   using C = Cfg<BN, CG, sizeof(TC)>;
@@ -533,7 +555,97 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
   const uint32_t tmem_base = *s_tmem;
   const int total = s_total;
 
-  if (warp == 0) {
+  if (warp == 0 && GATHER != 0) {
+    // ------------------------------------------------------------ producer (gathering, warp-wide)
+    int stage = 0;
+    uint32_t phase = 0;
+    int issued = 0;
+    uint32_t last_phase = 0;
+    int cur_g = -1;
+    bool ok = true;
+    for (int t = cta0; t < total && ok; t += ncta) {
+      Tile ti;
+      decode_tile<GROUP, CG>(p, t, s_off, s_pref, rank, ti);
+      const int64_t nb = ti.n0 * BN + (int64_t)rank * BNC;
+      int ra[4] = {0, 0, 0, 0};  // GATHER 1: source rows of this tile's rows 4 lane .. 4 lane + 3
+      if (GATHER == 1) {
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const int64_t r = ti.row0 + 4 * lane + i;
+          ra[i] = r < ti.row_end ? __ldg(p.gather + r) : 0;  // rows past the expert's end are dropped later
+        }
+      }
+      for (int kb = 0; kb < ti.nkb; ++kb) {
+        int okw = 1;
+        if (lane == 0) okw = wait_bounded<CG == 2>(smem_u32(&empty[stage]), phase ^ 1u, &s_abort, p.err) ? 1 : 0;
+        okw = __shfl_sync(0xffffffffu, okw, 0);
+        if (!okw) { ok = false; break; }
+        const uint32_t fb_local = smem_u32(&full[stage]);
+        const uint32_t fb = CG == 2 ? map_to_rank(fb_local, 0) : fb_local;
+        if (leader && lane == 0) mbar_expect_tx(fb_local, CG * C::kStageBytes);
+        __syncwarp();
+        const uint32_t sa = smem_u32(smem + stage * C::kStageBytes);
+        const uint32_t sb = sa + C::kABytes;
+        const int k0 = (int)(ti.kbeg + (int64_t)kb * BK);
+        auto load = [&](uint32_t dst, const CUtensorMap* m, int x, int y) {
+          if (CG == 2) tma_load_2d_pair(dst, m, fb, x, y);
+          else tma_load_2d(dst, m, fb, x, y);
+        };
+        auto gather4 = [&](uint32_t dst, const CUtensorMap* m, int x, const int* r) {
+          if (CG == 2) tma_gather4_pair(dst, m, fb, x, r[0], r[1], r[2], r[3]);
+          else tma_gather4(dst, m, fb, x, r[0], r[1], r[2], r[3]);
+        };
+        if (GATHER == 1) {
+          // A: the tile's 128 rows from the source, 4 per lane
+          gather4(sa + lane * 512, &p.ta, k0, ra);
+          if (lane == 0) {
+            if (B_MN) {
+              const int ky = (int)(ti.g * p.b_group_rows) + k0;
+#pragma unroll
+              for (int j = 0; j < BNC / 64; ++j) load(sb + j * 8192, &p.tb, (int)nb + 64 * j, ky);
+            } else {
+              load(sb, &p.tb, k0, (int)(ti.g * p.b_group_rows + nb));
+            }
+          }
+        } else {
+          // A from the group's own map (zero past the group's rows); B's 64 k
+          // rows from the source, in 64-column chunks of 16 four-row copies
+          if (lane == 0) {
+            const CUtensorMap* ma = p.gmaps + 2 * ti.g;
+            if (ti.g != cur_g) {
+              tmap_acquire(ma);
+              cur_g = ti.g;
+            }
+            const int ky = kb * BK;
+            load(sa, ma, (int)ti.row0, ky);
+            load(sa + 8192, ma, (int)ti.row0 + 64, ky);
+          }
+#pragma unroll
+          for (int u = lane; u < (BNC / 64) * 16; u += 32) {
+            const int j = u >> 4, qd = u & 15;
+            int rb[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              const int64_t kr = (int64_t)k0 + 4 * qd + i;
+              // past the group's rows A is zero, so any valid source row will do
+              rb[i] = kr < ti.kend ? __ldg(p.gather + kr) : 0;
+            }
+            gather4(sb + j * 8192 + qd * 512, &p.tb, (int)nb + 64 * j, rb);
+          }
+        }
+        last_phase = (last_phase & ~(1u << stage)) | (phase << stage);
+        ++issued;
+        if (++stage == C::kStages) { stage = 0; phase ^= 1u; }
+      }
+    }
+    if (leader && lane == 0) {
+      const int pending = issued < C::kStages ? issued : C::kStages;
+      for (int i = 0; i < pending; ++i) {
+        stage = (stage + C::kStages - 1) % C::kStages;
+        wait_drain<CG == 2>(smem_u32(&full[stage]), (last_phase >> stage) & 1u, 1000000000ull);
+      }
+    }
+  } else if (warp == 0) {
     // ------------------------------------------------------------ producer
     if (lane == 0) {
       int stage = 0;
@@ -879,16 +991,17 @@ __global__ void build_group_maps(const __grid_constant__ CUtensorMap ta, const _
   uint4* da = reinterpret_cast<uint4*>(ma);
   uint4* db = reinterpret_cast<uint4*>(mb);
 #pragma unroll
-  for (int i = 0; i < 8; ++i) {
-    da[i] = sa[i];
-    db[i] = sb[i];
-  }
+  for (int i = 0; i < 8; ++i) da[i] = sa[i];
   const uint64_t pa = reinterpret_cast<uint64_t>(a_base + lo * a_row_bytes);
-  const uint64_t pb = reinterpret_cast<uint64_t>(b_base + lo * b_row_bytes);
   asm volatile("tensormap.replace.tile.global_address.global.b1024.b64 [%0], %1;" ::"l"(ma), "l"(pa) : "memory");
   asm volatile("tensormap.replace.tile.global_dim.global.b1024.b32 [%0], 1, %1;" ::"l"(ma), "r"(dim) : "memory");
-  asm volatile("tensormap.replace.tile.global_address.global.b1024.b64 [%0], %1;" ::"l"(mb), "l"(pb) : "memory");
-  asm volatile("tensormap.replace.tile.global_dim.global.b1024.b32 [%0], 1, %1;" ::"l"(mb), "r"(dim) : "memory");
+  if (b_base) {  // NULL: B is gathered through one full map (no per-group B map)
+#pragma unroll
+    for (int i = 0; i < 8; ++i) db[i] = sb[i];
+    const uint64_t pb = reinterpret_cast<uint64_t>(b_base + lo * b_row_bytes);
+    asm volatile("tensormap.replace.tile.global_address.global.b1024.b64 [%0], %1;" ::"l"(mb), "l"(pb) : "memory");
+    asm volatile("tensormap.replace.tile.global_dim.global.b1024.b32 [%0], 1, %1;" ::"l"(mb), "r"(dim) : "memory");
+  }
   asm volatile("fence.proxy.tensormap::generic.release.gpu;" ::: "memory");
 }
 

@@ -136,6 +136,9 @@ struct GemmDesc {
                                      // (gemm_tc_group_scratch_bytes, 128-byte aligned)
   int64_t split_rows = 0;            // Group::K with offsets == nullptr: num_groups equal splits of
                                      // [0, split_rows) (split-K of a dense product)
+  const int32_t* gather = nullptr;   // row indirection into a source matrix of gather_rows rows:
+  int64_t gather_rows = 0;           //   Group::M: A's row m is source row gather[m];
+                                     //   Group::K: B's k row k is source row gather[k]
 };
 
 cudaError_t launch_gemm_simt(const Ctx& c, const GemmDesc& d, const char* name);

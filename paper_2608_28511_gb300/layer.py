@@ -26,13 +26,20 @@ class MoeLayer:
     enters the backward pass scaled by ``aux_grad``), Sec. 5.2.
     ``shared_F > 0`` adds the ungated shared expert of that width (Sec. 5.2),
     whose output is added to the layer output.
+    ``gather=True`` lets GEMM-1 and its weight gradient read the dispatched
+    rows straight from x by token_of_row (no x_perm copy, four-row TMA
+    gathers); the default ``False`` writes x_perm in the dispatch and reads it
+    back with tiled copies, which is faster on GB300 (a four-row gather of
+    128-byte rows moves far fewer bytes per copy-engine operation than a
+    128-row tile).
     """
 
     def __init__(self, S, GBS, K, D, E, F, dtype="bf16", H=0, device="cuda", router="softmax", aux_coef=1e-4,
-                 aux_grad=1.0, shared_F=0):
+                 aux_grad=1.0, shared_F=0, gather=False):
         if router not in ("softmax", "sigmoid"):
             raise ValueError(f"unknown router {router!r}")
         self.router = router
+        self.gather = bool(gather)
         self.aux_coef = float(aux_coef)
         self.aux_grad = float(aux_grad)
         self.shape = abi.MoeShape.of(S, GBS, K, D, E, F, dtype, H)
@@ -68,7 +75,7 @@ class MoeLayer:
         self.expert_offsets = e(E + 1, d=i32)
         self.row_of_slot = e(TK, d=i32)
         self.token_of_row = e(TK, d=i32)
-        self.x_perm = e(TK, D)
+        self.x_perm = None if self.gather else e(TK, D)
         self.prob_perm = e(TK, d=f32)
         self.h = e(TK, 2 * F)
         self.act = e(TK, F)
@@ -135,8 +142,12 @@ class MoeLayer:
             xd = self.x_lat
         abi.moe_dispatch(s, xd, self.topk_idx, self.topk_prob, self.expert_offsets, self.row_of_slot,
                          self.token_of_row, self.x_perm, self.prob_perm, self.ws, stream)
-        abi.moe_expert_ffn(s, self.x_perm, self.expert_offsets, self.w1, self.w2, self.h, self.act, self.y_perm,
-                           self.ws, stream)
+        if self.gather:
+            abi.moe_expert_ffn_gather(s, xd, self.token_of_row, self.expert_offsets, self.w1, self.w2, self.h,
+                                      self.act, self.y_perm, self.ws, stream)
+        else:
+            abi.moe_expert_ffn(s, self.x_perm, self.expert_offsets, self.w1, self.w2, self.h, self.act,
+                               self.y_perm, self.ws, stream)
         if self.H:
             abi.moe_combine(s, self.y_perm, self.prob_perm, self.row_of_slot, self.y_lat, stream)
             abi.moe_latent_proj(s, self.D, self.H, self.y_lat, self.w_upp, self.y, self.ws, stream)
@@ -156,8 +167,14 @@ class MoeLayer:
             dyd = self.dy_lat
         abi.moe_combine_bwd(s, dyd, self.y_perm, self.prob_perm, self.row_of_slot, self.dy_perm, self.dprob_perm,
                             stream)
-        abi.moe_expert_ffn_bwd(s, self.dy_perm, self.x_perm, self.h, self.act, self.expert_offsets, self.w1,
-                               self.w2, self.dx_perm, self.dw1, self.dw2, self.ws, stream)
+        if self.gather:
+            xd = self.x_lat if self.H else self.x
+            abi.moe_expert_ffn_bwd_gather(s, self.dy_perm, xd, self.token_of_row, self.h, self.act,
+                                          self.expert_offsets, self.w1, self.w2, self.dx_perm, self.dw1, self.dw2,
+                                          self.ws, stream)
+        else:
+            abi.moe_expert_ffn_bwd(s, self.dy_perm, self.x_perm, self.h, self.act, self.expert_offsets, self.w1,
+                                   self.w2, self.dx_perm, self.dw1, self.dw2, self.ws, stream)
         if self.H:
             abi.moe_dispatch_bwd(s, self.dx_perm, self.dprob_perm, self.row_of_slot, self.dx_lat, self.dprob, stream)
             abi.moe_latent_proj_bwd(s, self.H, self.D, self.dx_lat, self.x, self.w_down, self.dx, False,

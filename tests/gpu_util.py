@@ -32,13 +32,14 @@ def i64(t) -> np.ndarray:
     return t.detach().cpu().numpy().astype(np.int64)
 
 
-def make_layer(w: synth.Workload, T: int | None = None, seed: int | None = None, inputs: dict | None = None):
+def make_layer(w: synth.Workload, T: int | None = None, seed: int | None = None, inputs: dict | None = None,
+               gather: bool = False):
     """Build a MoeLayer for workload ``w`` (token count T), load seeded inputs, run forward+backward."""
     from paper_2608_28511_gb300.layer import MoeLayer
     T = w.T if T is None else T
     if inputs is None:
         inputs = synth.make_inputs(w, seed=seed, T=T)
-    layer = MoeLayer(T, 1, w.K, w.D, w.E, w.F, w.dtype, w.H)
+    layer = MoeLayer(T, 1, w.K, w.D, w.E, w.F, w.dtype, w.H, gather=gather)
     layer.load(inputs)
     layer.forward()
     layer.backward()

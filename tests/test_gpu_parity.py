@@ -1,5 +1,8 @@
 """GPU parity of every stage of the layer against the float64 oracle.
 
+The cached cases write x_perm (the default, as bench.py times it) so every
+stage is checked on its own; ``test_gpu_gather.py`` runs the gathering
+expert FFN and shows the two modes agree bit for bit.
 Stage-isolated checks feed the oracle the GPU's own inputs to that stage, so
 index work is compared bit for bit and float work within the layer's
 tolerances (relative Frobenius 1e-2, probabilities 1e-5 absolute, logits
