@@ -261,6 +261,8 @@ def main() -> None:
     ap.add_argument("--cpu-budget", type=float, default=15.0, help="seconds of CPU work for cpu_baseline")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=10)
+    ap.add_argument("--no-graph", action="store_true",
+                    help="launch every kernel from the host each step instead of replaying a captured CUDA graph")
     ap.add_argument("--shared-width", type=int, default=0,
                     help="hidden units of the ungated shared expert (0 = none; Sec. 5.2)")
     ap.add_argument("--router", default="softmax", choices=["softmax", "sigmoid"],
@@ -308,6 +310,12 @@ def main() -> None:
     torch.cuda.synchronize()
     assert abi.moe_check_device_status() == 0
 
+    graph = None
+    if not args.no_graph:
+        graph = L.capture()          # the step's launches, replayed as one graph
+        graph.replay()
+        torch.cuda.synchronize()
+
     def timed_steps(kernel_events: bool):
         """K steps, L2 flushed before each (outside the step events).  With
         kernel_events the library also brackets every kernel with CUDA events
@@ -322,10 +330,14 @@ def main() -> None:
         barrier()
         torch.cuda.synchronize()
         t0 = time.perf_counter()
+        use_graph = graph is not None and not kernel_events
         for i in range(args.steps):
             flush.zero_()
             ev_s[i].record(stream)
-            L.step()
+            if use_graph:
+                graph.replay()
+            else:
+                L.step()
             ev_e[i].record(stream)
         torch.cuda.synchronize()
         barrier()
@@ -337,11 +349,11 @@ def main() -> None:
         return step_ms, wall, launches, prof
 
     clocks = ClockSampler(local)
-    step_ms, wall, launches, _ = timed_steps(kernel_events=False)
+    step_ms, wall, _, _ = timed_steps(kernel_events=False)
     clk = clocks.stop()
     t_max = max_over_ranks(step_ms, world, "cuda")
     assert abi.moe_check_device_status() == 0
-    step_ms_ev, _, _, prof = timed_steps(kernel_events=True)
+    step_ms_ev, _, launches, prof = timed_steps(kernel_events=True)
     assert abi.moe_check_device_status() == 0
 
     # ---- end to end through the public API with host buffers
@@ -422,6 +434,7 @@ def main() -> None:
             "config": {"workload": w.name, "T": T, "S": w.S, "GBS": w.GBS, "D": w.D, "E": w.E, "K": w.K, "F": w.F,
                        "H": w.H, "seed": w.seed, "router": args.router, "shared_width": args.shared_width,
                        "parallelism": f"replicas x{world}, each rank its own tokens",
+                       "launch": "one CUDA graph per step" if graph is not None else "eager launches",
                        "l2": "256 MiB buffer written before every timed step (outside the step events); "
                              "the step also touches ~3 GB > 129 MB L2"},
             "roofline": roof,

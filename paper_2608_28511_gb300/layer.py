@@ -197,6 +197,17 @@ class MoeLayer:
         self.forward(stream)
         self.backward(stream)
 
+    def capture(self):
+        """Record one step (forward + backward) as a CUDA graph.  Every entry
+        point only enqueues kernels on the current stream, with buffers and
+        workspace allocated up front, so the step is capturable; replay() then
+        runs the same launches without per-launch host work.  Run one eager
+        step first (it sets up per-kernel attributes)."""
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            self.step()
+        return g
+
     # ------------------------------------------------------------------
     def unpack_w1_like(self, t: torch.Tensor):
         """Split a packed [E, 2F, D] tensor (w1 or dw1) into gate and up [E, F, D]."""

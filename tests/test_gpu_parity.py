@@ -261,3 +261,20 @@ def test_out_of_range_expert_index_sets_status_word():
     assert abi.moe_check_device_status() == -7
     assert abi.moe_check_device_status() == 0      # cleared
     assert int(off[-1]) == 126                     # only valid slots are counted
+
+
+def test_graph_replay_matches_eager_bitwise():
+    """A captured CUDA graph of the step (as bench.py replays it) reproduces the eager step bit for bit."""
+    w = CASES["mid_skew"]
+    inp = synth.make_inputs(w)
+    L, _ = make_layer(w, inputs=inp)
+    names = ("topk_idx", "topk_prob", "row_of_slot", "x_perm", "h", "act", "y_perm", "y", "dy_perm", "dprob_perm",
+             "dx_perm", "dw1", "dw2", "dx", "dlogits", "dw_router")
+    eager = {n: getattr(L, n).clone() for n in names}
+    g = L.capture()
+    for n in names:
+        getattr(L, n).zero_()
+    g.replay()
+    torch.cuda.synchronize()
+    for n in names:
+        assert torch.equal(getattr(L, n), eager[n]), n
