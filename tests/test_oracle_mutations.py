@@ -177,3 +177,32 @@ def test_shared_expert_mistakes_are_caught(monkeypatch):
     monkeypatch.setattr(SE, "shared_expert", transposed_down)
     monkeypatch.setattr(oracle, "shared_expert", transposed_down)
     _expect_failure(PSH.test_forward_is_a_sum_of_squared_positive_projections)
+
+
+def test_fp8_payload_mistakes_are_caught(monkeypatch):
+    import oracle.fp8 as F
+    import tests.test_oracle_fp8 as PF
+
+    def ties_away(v):
+        neg = v < 0
+        a = abs(v)
+        if a >= F.E4M3_MAX:
+            return F._CODES[-1] | (0x80 if neg else 0)
+        best = min(zip(F._CODES, F._VALS), key=lambda cv: (abs(cv[1] - a), -cv[1]))   # ties to the larger
+        return best[0] | (0x80 if neg else 0)
+    monkeypatch.setattr(F, "e4m3_quantize", ties_away)
+    monkeypatch.setattr(oracle, "e4m3_quantize", ties_away)
+    _expect_failure(PF.test_ties_go_to_the_even_code_and_saturate)
+    monkeypatch.undo()
+
+    def scale_one_too_big(row):
+        amax = float(np.max(np.abs(row)))
+        if amax == 0.0:
+            return 1.0
+        e = -126
+        while amax > F.E4M3_MAX * 2.0 ** e:
+            e += 1
+        return 2.0 ** (e + 1)                              # not the smallest fitting power of two
+    monkeypatch.setattr(F, "fp8_row_scale", scale_one_too_big)
+    monkeypatch.setattr(oracle, "fp8_row_scale", scale_one_too_big)
+    _expect_failure(PF.test_row_scale_is_the_smallest_fitting_power_of_two)
