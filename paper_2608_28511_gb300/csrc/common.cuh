@@ -19,18 +19,6 @@ __device__ __forceinline__ void set_error(uint32_t* err, uint32_t bit) {
   if (err) atomicOr(err, bit);
 }
 
-// Programmatic dependent launch.  Every kernel of the library calls this
-// before its first global-memory access: it waits until the grids it depends
-// on in the stream have completed and their writes are visible (a no-op when
-// the kernel was launched without the attribute), then lets the next grid in
-// the stream begin launching.  That grid is released only once every CTA of
-// this one has started, so its waiting CTAs never hold resources this grid
-// still needs.
-__device__ __forceinline__ void pdl_enter() {
-  asm volatile("griddepcontrol.wait;" ::: "memory");
-  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-}
-
 // ---- conversions -----------------------------------------------------------
 template <typename T> __device__ __forceinline__ float to_f32(T v);
 template <> __device__ __forceinline__ float to_f32<float>(float v) { return v; }

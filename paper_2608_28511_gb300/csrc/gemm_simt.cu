@@ -25,7 +25,6 @@ __device__ __forceinline__ float silu_f(float v) { return v / (1.0f + __expf(-v)
 
 template <typename TA, typename TB, typename TC>
 __global__ void __launch_bounds__(256) simt_gemm_kernel(GemmDesc d) {
-  pdl_enter();
   __shared__ float As[BK][BM + 4];
   __shared__ float Bs[BK][BN + 4];
   const int tid = threadIdx.x;
@@ -168,7 +167,7 @@ cudaError_t run(const Ctx& c, const GemmDesc& d) {
     grid.y = (unsigned)((d.M + BM - 1) / BM);
   }
   if (grid.x == 0 || grid.y == 0 || grid.z == 0) return cudaSuccess;
-  launch_pdl(simt_gemm_kernel<TA, TB, TC>, grid, block, 0, c.stream, d);
+  simt_gemm_kernel<TA, TB, TC><<<grid, block, 0, c.stream>>>(d);
   return cudaGetLastError();
 }
 

@@ -145,7 +145,7 @@ cudaError_t launch_inst(const Ctx& c, const Params& p, int64_t ub) {
   }
   if (CG == 1) {
     const int grid = (int)(ub < c.num_sms ? ub : c.num_sms);
-    launch_pdl(k, grid, kThreads, kSmem, c.stream, p);
+    k<<<grid, kThreads, kSmem, c.stream>>>(p);
     return cudaGetLastError();
   }
   int np = pairs > 0 ? pairs : c.num_sms / 2;
@@ -155,15 +155,13 @@ cudaError_t launch_inst(const Ctx& c, const Params& p, int64_t ub) {
   cfg.blockDim = dim3(kThreads, 1, 1);
   cfg.dynamicSmemBytes = kSmem;
   cfg.stream = c.stream;
-  cudaLaunchAttribute attr[2];
+  cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = 2;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
-  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;  // see launch_pdl
-  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 2;
+  cfg.numAttrs = 1;
   return cudaLaunchKernelEx(&cfg, k, p);
 }
 
@@ -246,7 +244,7 @@ cudaError_t launch_gemm_tc(const Ctx& c, const GemmDesc& d, const char* name) {
     int32_t* split_offs = d.offsets ? nullptr : reinterpret_cast<int32_t*>(maps + 2 * d.num_groups);
     {
       KernelScope ks("group_maps", c.stream);
-      launch_pdl(tc::build_group_maps, (d.num_groups + 127) / 128, 128, 0, c.stream, 
+      tc::build_group_maps<<<(d.num_groups + 127) / 128, 128, 0, c.stream>>>(
           p.ta, p.tb, d.offsets, d.num_groups, d.split_rows, split_offs, static_cast<const uint8_t*>(d.A),
           pl.lda * 2, gb ? nullptr : static_cast<const uint8_t*>(d.B), pl.ldb * 2, maps);
     }

@@ -529,7 +529,6 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
     tmem_alloc_cg<CG>(smem_u32(s_tmem), C::kCols);
     tmem_relinquish_cg<CG>();
   }
-  pdl_enter();  // the barriers and TMEM above overlap the previous kernel's tail
   if (GROUP != 0) {
     for (int i = tid; i <= p.num_groups; i += C::kThreads) s_off[i] = p.offsets[i];
   }
@@ -971,7 +970,6 @@ __global__ void build_group_maps(const __grid_constant__ CUtensorMap ta, const _
                                  const int32_t* __restrict__ offsets, int G, int64_t split_rows,
                                  int32_t* __restrict__ offs_out, const uint8_t* a_base, int64_t a_row_bytes,
                                  const uint8_t* b_base, int64_t b_row_bytes, CUtensorMap* out) {
-  pdl_enter();
   const int g = blockIdx.x * blockDim.x + threadIdx.x;
   if (g >= G) return;
   int64_t lo, hi;

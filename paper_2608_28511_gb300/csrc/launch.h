@@ -28,26 +28,6 @@ struct KernelScope {
   ~KernelScope() { prof_end(name, s); count_launch(); }
 };
 
-// Launches kernel<<<grid, block, smem, stream>>>(args...) with programmatic
-// stream serialization, so its launch and prologue may overlap the tail of
-// the previous kernel in the stream (each kernel synchronises through
-// pdl_enter before touching global memory).
-template <typename... KArgs, typename... Args>
-cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t stream,
-                       Args&&... args) {
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = grid;
-  cfg.blockDim = block;
-  cfg.dynamicSmemBytes = smem;
-  cfg.stream = stream;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args&&>(args)...);
-}
-
 enum class DType : int { BF16 = 0, F32 = 1 };
 
 inline size_t dsize(DType t) { return t == DType::BF16 ? 2 : 4; }

@@ -22,7 +22,6 @@ size_t perm_workspace_bytes(int64_t TK, int E) {
 // so the result is deterministic).  Layout: counts[e * nchunks + chunk].
 __global__ void __launch_bounds__(256) perm_hist_kernel(const int32_t* __restrict__ idx, int64_t TK, int E,
                                                         int nchunks, int32_t* __restrict__ counts, uint32_t* err) {
-  pdl_enter();
   __shared__ int h[kMaxE];
   for (int i = threadIdx.x; i < E; i += blockDim.x) h[i] = 0;
   __syncthreads();
@@ -42,7 +41,6 @@ __global__ void __launch_bounds__(256) perm_hist_kernel(const int32_t* __restric
 // offsets[e] = base[e * nchunks], offsets[E] = number of valid slots.
 __global__ void __launch_bounds__(1024) perm_scan_kernel(const int32_t* __restrict__ counts, int E, int nchunks,
                                                          int32_t* __restrict__ base, int32_t* __restrict__ offsets) {
-  pdl_enter();
   __shared__ int part[1024];
   const int n = E * nchunks;
   const int per = (n + 1023) / 1024;
@@ -76,7 +74,6 @@ __global__ void __launch_bounds__(kRankWarps * 32) perm_rank_kernel(
     const int32_t* __restrict__ idx, const float* __restrict__ prob, int64_t TK, int K, int E, int nchunks,
     const int32_t* __restrict__ base, int32_t* __restrict__ row_of_slot, int32_t* __restrict__ token_of_row,
     float* __restrict__ prob_perm) {
-  pdl_enter();
   __shared__ int cnt[kRankWarps * kMaxE];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   for (int i = threadIdx.x; i < kRankWarps * E; i += blockDim.x) cnt[i] = 0;
@@ -134,19 +131,19 @@ cudaError_t launch_permutation(const Ctx& c, const int32_t* idx, const float* pr
   }
   {
     KernelScope ks("perm_hist", c.stream);
-    launch_pdl(perm_hist_kernel, nch, 256, 0, c.stream, idx, TK, E, nch, counts, c.err);
+    perm_hist_kernel<<<nch, 256, 0, c.stream>>>(idx, TK, E, nch, counts, c.err);
   }
   cudaError_t st = cudaGetLastError();
   if (st != cudaSuccess) return st;
   {
     KernelScope ks("perm_scan", c.stream);
-    launch_pdl(perm_scan_kernel, 1, 1024, 0, c.stream, counts, E, nch, base, offsets);
+    perm_scan_kernel<<<1, 1024, 0, c.stream>>>(counts, E, nch, base, offsets);
   }
   st = cudaGetLastError();
   if (st != cudaSuccess) return st;
   {
     KernelScope ks("perm_rank", c.stream);
-    launch_pdl(perm_rank_kernel, nch, kRankWarps * 32, 0, c.stream, idx, prob, TK, K, E, nch, base, row_of_slot,
+    perm_rank_kernel<<<nch, kRankWarps * 32, 0, c.stream>>>(idx, prob, TK, K, E, nch, base, row_of_slot,
                                                             token_of_row, prob_perm);
   }
   return cudaGetLastError();
@@ -180,7 +177,6 @@ template <int KM>
 __global__ void __launch_bounds__(256) dispatch_rows_kernel(const uint4* __restrict__ x,
                                                             const int32_t* __restrict__ row_of_slot, int64_t T,
                                                             int K, int vpr, uint4* __restrict__ x_perm) {
-  pdl_enter();
   const int lane = threadIdx.x & 31;
   const int64_t t = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   if (t >= T) return;
@@ -202,7 +198,7 @@ cudaError_t launch_dispatch_rows(const Ctx& c, const void* x, const int32_t* row
   const unsigned grid = (unsigned)((T + warps - 1) / warps);
   const int vpr = (int)(row_bytes / 16);
   KernelScope ks("dispatch_rows", c.stream);
-  MOE_DISPATCH_KM(K, (launch_pdl(dispatch_rows_kernel<KM>, grid, 32 * warps, 0, c.stream, 
+  MOE_DISPATCH_KM(K, (dispatch_rows_kernel<KM><<<grid, 32 * warps, 0, c.stream>>>(
                          (const uint4*)x, row_of_slot, T, K, vpr, (uint4*)x_perm)));
   return cudaGetLastError();
 }
@@ -213,7 +209,6 @@ __global__ void __launch_bounds__(256) combine_kernel(const uint4* __restrict__ 
                                                       const float* __restrict__ prob_perm,
                                                       const int32_t* __restrict__ row_of_slot, int64_t Tn, int K,
                                                       int vpr, uint4* __restrict__ y) {
-  pdl_enter();
   constexpr int NV = Vec<T>::N;
   const int lane = threadIdx.x & 31;
   const int64_t t = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
@@ -252,10 +247,10 @@ cudaError_t launch_combine(const Ctx& c, DType dt, const void* y_perm, const flo
   const unsigned grid = (unsigned)((T + warps - 1) / warps);
   KernelScope ks("combine", c.stream);
   if (dt == DType::BF16) {
-    MOE_DISPATCH_KM(K, (launch_pdl(combine_kernel<bf16, KM>, grid, 32 * warps, 0, c.stream, 
+    MOE_DISPATCH_KM(K, (combine_kernel<bf16, KM><<<grid, 32 * warps, 0, c.stream>>>(
                            (const uint4*)y_perm, prob_perm, row_of_slot, T, K, vpr, (uint4*)y)));
   } else {
-    MOE_DISPATCH_KM(K, (launch_pdl(combine_kernel<float, KM>, grid, 32 * warps, 0, c.stream, 
+    MOE_DISPATCH_KM(K, (combine_kernel<float, KM><<<grid, 32 * warps, 0, c.stream>>>(
                            (const uint4*)y_perm, prob_perm, row_of_slot, T, K, vpr, (uint4*)y)));
   }
   return cudaGetLastError();
@@ -269,7 +264,6 @@ __global__ void __launch_bounds__(256) combine_bwd_kernel(const uint4* __restric
                                                           const int32_t* __restrict__ row_of_slot, int64_t Tn,
                                                           int K, int vpr, uint4* __restrict__ dy_perm,
                                                           float* __restrict__ dprob_perm) {
-  pdl_enter();
   constexpr int NV = Vec<T>::N;
   const int lane = threadIdx.x & 31;
   const int64_t t = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
@@ -324,11 +318,11 @@ cudaError_t launch_combine_bwd(const Ctx& c, DType dt, const void* dy, const voi
   const unsigned grid = (unsigned)((T + warps - 1) / warps);
   KernelScope ks("combine_bwd", c.stream);
   if (dt == DType::BF16) {
-    MOE_DISPATCH_KM(K, (launch_pdl(combine_bwd_kernel<bf16, KM>, grid, 32 * warps, 0, c.stream, 
+    MOE_DISPATCH_KM(K, (combine_bwd_kernel<bf16, KM><<<grid, 32 * warps, 0, c.stream>>>(
                            (const uint4*)dy, (const uint4*)y_perm, prob_perm, row_of_slot, T, K, vpr,
                            (uint4*)dy_perm, dprob_perm)));
   } else {
-    MOE_DISPATCH_KM(K, (launch_pdl(combine_bwd_kernel<float, KM>, grid, 32 * warps, 0, c.stream, 
+    MOE_DISPATCH_KM(K, (combine_bwd_kernel<float, KM><<<grid, 32 * warps, 0, c.stream>>>(
                            (const uint4*)dy, (const uint4*)y_perm, prob_perm, row_of_slot, T, K, vpr,
                            (uint4*)dy_perm, dprob_perm)));
   }
@@ -343,7 +337,6 @@ __global__ void __launch_bounds__(256) dispatch_bwd_kernel(const uint4* __restri
                                                            const int32_t* __restrict__ row_of_slot, int64_t Tn,
                                                            int K, int vpr, uint4* __restrict__ dx,
                                                            float* __restrict__ dprob) {
-  pdl_enter();
   constexpr int NV = Vec<T>::N;
   const int lane = threadIdx.x & 31;
   const int64_t t = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
@@ -380,10 +373,10 @@ cudaError_t launch_dispatch_bwd(const Ctx& c, DType dt, const void* dx_perm, con
   const unsigned grid = (unsigned)((T + warps - 1) / warps);
   KernelScope ks("dispatch_bwd", c.stream);
   if (dt == DType::BF16) {
-    MOE_DISPATCH_KM(K, (launch_pdl(dispatch_bwd_kernel<bf16, KM>, grid, 32 * warps, 0, c.stream, 
+    MOE_DISPATCH_KM(K, (dispatch_bwd_kernel<bf16, KM><<<grid, 32 * warps, 0, c.stream>>>(
                            (const uint4*)dx_perm, dprob_perm, row_of_slot, T, K, vpr, (uint4*)dx, dprob)));
   } else {
-    MOE_DISPATCH_KM(K, (launch_pdl(dispatch_bwd_kernel<float, KM>, grid, 32 * warps, 0, c.stream, 
+    MOE_DISPATCH_KM(K, (dispatch_bwd_kernel<float, KM><<<grid, 32 * warps, 0, c.stream>>>(
                            (const uint4*)dx_perm, dprob_perm, row_of_slot, T, K, vpr, (uint4*)dx, dprob)));
   }
   return cudaGetLastError();
@@ -392,7 +385,6 @@ cudaError_t launch_dispatch_bwd(const Ctx& c, DType dt, const void* dx_perm, con
 // w1[e, 128 i + c] = w_gate[e, 64 i + c] for c < 64, w_up[e, 64 i + c - 64] otherwise.
 __global__ void __launch_bounds__(256) pack_w1_kernel(const uint4* __restrict__ wg, const uint4* __restrict__ wu,
                                                       int64_t rows_total, int F, int vpr, uint4* __restrict__ w1) {
-  pdl_enter();
   const int64_t r = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   if (r >= rows_total) return;
   const int lane = threadIdx.x & 31;
@@ -409,7 +401,7 @@ cudaError_t launch_pack_w1(const Ctx& c, DType dt, const void* w_gate, const voi
   const int64_t rows = (int64_t)E * 2 * F;
   const int vpr = (int)((int64_t)D * dsize(dt) / 16);
   KernelScope ks("pack_w1", c.stream);
-  launch_pdl(pack_w1_kernel, (unsigned)((rows + 7) / 8), 256, 0, c.stream, (const uint4*)w_gate, (const uint4*)w_up, rows,
+  pack_w1_kernel<<<(unsigned)((rows + 7) / 8), 256, 0, c.stream>>>((const uint4*)w_gate, (const uint4*)w_up, rows,
                                                                    F, vpr, (uint4*)w1);
   return cudaGetLastError();
 }

@@ -19,7 +19,6 @@ struct Identity {
 template <int KM>
 __global__ void __launch_bounds__(256) topk_kernel(const float* __restrict__ logits, int64_t T, int E, int K,
                                                    int tpb, int32_t* __restrict__ idx, float* __restrict__ prob) {
-  pdl_enter();
   extern __shared__ __align__(16) float zs[];  // [tpb][E]
   const int tid = threadIdx.x;
   const int64_t t0 = (int64_t)blockIdx.x * tpb;
@@ -61,10 +60,10 @@ cudaError_t launch_topk(const Ctx& c, const float* logits, int64_t T, int E, int
   const size_t smem = (size_t)tpb * E * 4;
   KernelScope ks("topk", c.stream);
   switch (sel::k_bound(K)) {
-    case 2: launch_pdl(topk_kernel<2>, grid, 4 * tpb, smem, c.stream, logits, T, E, K, tpb, idx, prob); break;
-    case 4: launch_pdl(topk_kernel<4>, grid, 4 * tpb, smem, c.stream, logits, T, E, K, tpb, idx, prob); break;
-    case 8: launch_pdl(topk_kernel<8>, grid, 4 * tpb, smem, c.stream, logits, T, E, K, tpb, idx, prob); break;
-    default: launch_pdl(topk_kernel<16>, grid, 4 * tpb, smem, c.stream, logits, T, E, K, tpb, idx, prob); break;
+    case 2: topk_kernel<2><<<grid, 4 * tpb, smem, c.stream>>>(logits, T, E, K, tpb, idx, prob); break;
+    case 4: topk_kernel<4><<<grid, 4 * tpb, smem, c.stream>>>(logits, T, E, K, tpb, idx, prob); break;
+    case 8: topk_kernel<8><<<grid, 4 * tpb, smem, c.stream>>>(logits, T, E, K, tpb, idx, prob); break;
+    default: topk_kernel<16><<<grid, 4 * tpb, smem, c.stream>>>(logits, T, E, K, tpb, idx, prob); break;
   }
   return cudaGetLastError();
 }
@@ -75,7 +74,6 @@ __global__ void __launch_bounds__(256) route_dz_kernel(const int32_t* __restrict
                                                        const float* __restrict__ prob,
                                                        const float* __restrict__ dprob, int64_t T, int E, int K,
                                                        float* __restrict__ dz, bf16* __restrict__ dz_bf16) {
-  pdl_enter();
   const int lane = threadIdx.x & 31;
   const int64_t t = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   if (t >= T) return;
@@ -111,7 +109,7 @@ cudaError_t launch_route_dz(const Ctx& c, const int32_t* idx, const float* prob,
   const int warps = 8;
   dim3 grid((unsigned)((T + warps - 1) / warps)), block(32 * warps);
   KernelScope ks("route_dz", c.stream);
-  launch_pdl(route_dz_kernel, grid, block, 0, c.stream, idx, prob, dprob, T, E, K, dz, (bf16*)dz_bf16);
+  route_dz_kernel<<<grid, block, 0, c.stream>>>(idx, prob, dprob, T, E, K, dz, (bf16*)dz_bf16);
   return cudaGetLastError();
 }
 
@@ -119,7 +117,6 @@ cudaError_t launch_route_dz(const Ctx& c, const int32_t* idx, const float* prob,
 // in-order sum of its S partials.
 __global__ void __launch_bounds__(256) sum_splits_kernel(const float4* __restrict__ part, int S, int64_t n4,
                                                          float4* __restrict__ out) {
-  pdl_enter();
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n4; i += (int64_t)gridDim.x * blockDim.x) {
     float4 a = __ldcs(part + i);
     for (int s = 1; s < S; ++s) {
@@ -138,7 +135,7 @@ cudaError_t launch_sum_splits(const Ctx& c, const float* part, int S, int64_t n,
   const int64_t want = (n4 + 255) / 256;
   const int blocks = (int)(want < (int64_t)c.num_sms * 8 ? want : (int64_t)c.num_sms * 8);
   KernelScope ks("sum_splits", c.stream);
-  launch_pdl(sum_splits_kernel, blocks, 256, 0, c.stream, (const float4*)part, S, n4, (float4*)out);
+  sum_splits_kernel<<<blocks, 256, 0, c.stream>>>((const float4*)part, S, n4, (float4*)out);
   return cudaGetLastError();
 }
 

@@ -37,7 +37,6 @@ __global__ void __launch_bounds__(256) select_sigmoid_kernel(
     const float* __restrict__ logits, const float* __restrict__ bias, int64_t S, int E, int K, int tpb, int nch,
     int32_t* __restrict__ idx, float* __restrict__ prob, float* __restrict__ psum, int32_t* __restrict__ pcnt,
     uint32_t* __restrict__ ticket) {
-  pdl_enter();
   extern __shared__ __align__(16) float sm[];
   float* zs = sm;                                   // [tpb][E] scores
   float* bs = zs + tpb * E;                         // [E]
@@ -97,7 +96,6 @@ __global__ void __launch_bounds__(256) balance_finalize_kernel(const float* __re
                                                                float* __restrict__ f_out, float* __restrict__ tile_sum,
                                                                uint32_t* __restrict__ ticket,
                                                                float* __restrict__ loss) {
-  pdl_enter();
   __shared__ float rp[8][32];
   __shared__ int rc[8][32];
   const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
@@ -158,7 +156,6 @@ __global__ void __launch_bounds__(256) route_dz_sigmoid_kernel(
     const float* __restrict__ logits, const int32_t* __restrict__ idx, const float* __restrict__ prob,
     const float* __restrict__ dprob, const float* __restrict__ f, int64_t T, int64_t S, int E, int K, float cscale,
     float* __restrict__ dz, bf16* __restrict__ dz16, uint32_t* err) {
-  pdl_enter();
   const int lane = threadIdx.x & 31;
   const int64_t t = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   if (t >= T) return;
@@ -258,7 +255,7 @@ cudaError_t launch_route_sigmoid_select(const Ctx& c, const float* logits, const
     dim3 grid((unsigned)nch, (unsigned)GBS);
     KernelScope ks("select_sigmoid", c.stream);
 #define MOE_SELECT_SIGMOID(KM)                                                                             \
-  launch_pdl(select_sigmoid_kernel<KM>, grid, 4 * tpb, smem, c.stream, logits, bias, S, E, K, tpb, (int)nch, idx, \
+  select_sigmoid_kernel<KM><<<grid, 4 * tpb, smem, c.stream>>>(logits, bias, S, E, K, tpb, (int)nch, idx, \
                                                                prob, psum, pcnt, ticket)
     switch (sel::k_bound(K)) {
       case 2: MOE_SELECT_SIGMOID(2); break;
@@ -273,7 +270,7 @@ cudaError_t launch_route_sigmoid_select(const Ctx& c, const float* logits, const
   {
     KernelScope ks("balance_finalize", c.stream);
     dim3 grid((unsigned)((E + 31) / 32), (unsigned)GBS);
-    launch_pdl(balance_finalize_kernel, grid, 256, 0, c.stream, psum, pcnt, S, E, K, (int)nch, coef, (int)GBS, f_out,
+    balance_finalize_kernel<<<grid, 256, 0, c.stream>>>(psum, pcnt, S, E, K, (int)nch, coef, (int)GBS, f_out,
                                                         tile_sum, ticket, loss);
   }
   return cudaGetLastError();
@@ -289,7 +286,7 @@ cudaError_t launch_route_dz_sigmoid(const Ctx& c, const float* logits, const int
   bf16* d16 = static_cast<bf16*>(dz16);
   KernelScope ks("route_dz_sigmoid", c.stream);
 #define MOE_DZ_SIGMOID(VPL)                                                                                     \
-  launch_pdl(route_dz_sigmoid_kernel<VPL>, grid, block, 0, c.stream, logits, idx, prob, dprob, f, T, S, E, K, cscale, dz, \
+  route_dz_sigmoid_kernel<VPL><<<grid, block, 0, c.stream>>>(logits, idx, prob, dprob, f, T, S, E, K, cscale, dz, \
                                                              d16, c.err)
   const int vpl = (E + 31) / 32;
   if (vpl <= 1) MOE_DZ_SIGMOID(1);

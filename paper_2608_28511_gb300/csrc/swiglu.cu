@@ -12,7 +12,6 @@ namespace moe {
 template <typename T>
 __global__ void __launch_bounds__(256) swiglu_bwd_kernel(const uint4* __restrict__ dA, const T* __restrict__ h,
                                                          int64_t rows, int F, T* __restrict__ dH) {
-  pdl_enter();
   constexpr int NV = Vec<T>::N;
   const int64_t vpr = F / NV;  // 16-byte vectors of dA per row
   const int64_t total = rows * vpr;
@@ -44,9 +43,9 @@ cudaError_t launch_swiglu_bwd(const Ctx& c, DType dt, const void* dA, const void
   const int blocks = (int)(want < (int64_t)c.num_sms * 16 ? want : (int64_t)c.num_sms * 16);
   KernelScope ks("swiglu_bwd", c.stream);
   if (dt == DType::BF16)
-    launch_pdl(swiglu_bwd_kernel<bf16>, blocks, 256, 0, c.stream, (const uint4*)dA, (const bf16*)h, rows, F, (bf16*)dH);
+    swiglu_bwd_kernel<bf16><<<blocks, 256, 0, c.stream>>>((const uint4*)dA, (const bf16*)h, rows, F, (bf16*)dH);
   else
-    launch_pdl(swiglu_bwd_kernel<float>, blocks, 256, 0, c.stream, (const uint4*)dA, (const float*)h, rows, F,
+    swiglu_bwd_kernel<float><<<blocks, 256, 0, c.stream>>>((const uint4*)dA, (const float*)h, rows, F,
                                                            (float*)dH);
   return cudaGetLastError();
 }
@@ -56,7 +55,6 @@ cudaError_t launch_swiglu_bwd(const Ctx& c, DType dt, const void* dA, const void
 template <typename T>
 __global__ void __launch_bounds__(256) relusq_bwd_kernel(const uint4* dA, const uint4* __restrict__ h, int64_t nvec,
                                                          uint4* dh) {
-  pdl_enter();
   constexpr int NV = Vec<T>::N;
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < nvec; i += (int64_t)gridDim.x * blockDim.x) {
     float a[NV], hv[NV];
@@ -75,9 +73,9 @@ cudaError_t launch_relusq_bwd(const Ctx& c, DType dt, const void* dA, const void
   const int blocks = (int)(want < (int64_t)c.num_sms * 16 ? want : (int64_t)c.num_sms * 16);
   KernelScope ks("relusq_bwd", c.stream);
   if (dt == DType::BF16)
-    launch_pdl(relusq_bwd_kernel<bf16>, blocks, 256, 0, c.stream, (const uint4*)dA, (const uint4*)h, vecs, (uint4*)dh);
+    relusq_bwd_kernel<bf16><<<blocks, 256, 0, c.stream>>>((const uint4*)dA, (const uint4*)h, vecs, (uint4*)dh);
   else
-    launch_pdl(relusq_bwd_kernel<float>, blocks, 256, 0, c.stream, (const uint4*)dA, (const uint4*)h, vecs, (uint4*)dh);
+    relusq_bwd_kernel<float><<<blocks, 256, 0, c.stream>>>((const uint4*)dA, (const uint4*)h, vecs, (uint4*)dh);
   return cudaGetLastError();
 }
 
