@@ -343,7 +343,6 @@ __global__ void __launch_bounds__(256) dispatch_bwd_kernel(const uint4* __restri
   if (t >= Tn) return;
   int32_t rows[KM];
   load_rows<KM>(row_of_slot, t, K, rows);
-  if (lane < K) dprob[t * K + lane] = __ldg(dprob_perm + row_of_slot[t * K + lane]);
   for (int v = lane; v < vpr; v += 32) {
     uint4 raw[KM];
 #pragma unroll
@@ -363,6 +362,8 @@ __global__ void __launch_bounds__(256) dispatch_bwd_kernel(const uint4* __restri
     }
     st_stream(dx + t * vpr + v, pack16<T>(acc));
   }
+  // the probability gradients last, off the path of the row loads
+  if (lane < K) dprob[t * K + lane] = __ldg(dprob_perm + row_of_slot[t * K + lane]);
 }
 
 cudaError_t launch_dispatch_bwd(const Ctx& c, DType dt, const void* dx_perm, const float* dprob_perm,
