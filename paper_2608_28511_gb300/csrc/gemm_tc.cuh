@@ -399,14 +399,7 @@ struct Tile {
   int g;
   int64_t row0, row_end, n0, kbeg, kend;
   int nkb;
-  bool half;  // CTA pair, Group::M: a group's last <= 128 rows as one M = 128 MMA (64 rows per CTA)
 };
-
-// Accumulator of a half tile (M = 128 on a CTA pair: 64 rows per CTA, a
-// measured layout): row i, column n < BN/2 sits in TMEM lane i, column n; row
-// i, column n >= BN/2 in lane 64 + i, column n - BN/2.  So lane quarters 0, 1
-// hold rows 0..63 of the left half of the columns, quarters 2, 3 the same rows
-// of the right half.
 
 // Tile t of the static sequence.  GROUP: 0 dense, 1 by M, 2 by K.  Tiles
 // are BM * CG rows high; row0 is this CTA's first row (rank * BM into the tile).
@@ -414,7 +407,6 @@ template <int GROUP, int CG = 1>
 __device__ __forceinline__ void decode_tile(const Params& p, int t, const int* s_off, const int* s_pref,
                                             uint32_t rank, Tile& ti) {
   constexpr int BMP = BM * CG;
-  ti.half = false;
   if (GROUP == 0) {
     const int mt = t / p.tiles_n, nt = t % p.tiles_n;
     ti.g = 0;
@@ -432,11 +424,7 @@ __device__ __forceinline__ void decode_tile(const Params& p, int t, const int* s
       else hi = mid - 1;
     }
     ti.g = lo;
-    const int j = mb - s_pref[lo];
-    const int rows = s_off[lo + 1] - s_off[lo];
-    // a pair's last tile of a group whose rows past its full 256-row tiles fit in 128
-    ti.half = CG == 2 && j == rows / BMP && rows % BMP != 0 && rows % BMP <= BMP / 2;
-    ti.row0 = (int64_t)s_off[lo] + (int64_t)j * BMP + rank * (ti.half ? BM / 2 : BM);
+    ti.row0 = (int64_t)s_off[lo] + (int64_t)(mb - s_pref[lo]) * BMP + rank * BM;
     ti.row_end = s_off[lo + 1];
     ti.n0 = nt;
     ti.kbeg = 0;
@@ -502,7 +490,6 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
   constexpr int BMP = BM * CG;
   constexpr int BNC = C::kBRows;
   constexpr uint32_t kIdesc = make_idesc(BN, BMP, A_MN, B_MN);
-  constexpr uint32_t kIdescHalf = make_idesc(BN, BMP / 2, A_MN, B_MN);  // half tiles (CG 2 only)
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::kStages * C::kStageBytes + C::kStagingBytes);
@@ -760,7 +747,7 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
             else ad = make_sdesc(sa + k * 32, 16, 1024);
             if (B_MN) bd = make_sdesc(sb + k * 2048, 8192, 1024);
             else bd = make_sdesc(sb + k * 32, 16, 1024);
-            mma_bf16_cg<CG>(d_tmem, ad, bd, ti.half ? kIdescHalf : kIdesc, (kb > 0 || k > 0) ? 1u : 0u);
+            mma_bf16_cg<CG>(d_tmem, ad, bd, kIdesc, (kb > 0 || k > 0) ? 1u : 0u);
           }
           mma_commit_cg<CG>(smem_u32(&empty[stage]), kBoth);
         }
@@ -795,10 +782,7 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
       Tile ti;
       decode_tile<GROUP, CG>(p, t, s_off, s_pref, rank, ti);
       const int64_t n0 = ti.n0 * BN;
-      // this warp's first row and row count (its lane quarter holds 32 rows; in a
-      // half tile quarters q and q + 2 hold the same rows, for the two column halves)
-      const int hsel = ti.half ? (q >> 1) : -1;  // half tile: the column half this quarter holds
-      const int64_t rbase = ti.row0 + (ti.half ? (q & 1) : q) * 32;
+      const int64_t rbase = ti.row0 + q * 32;  // this warp's first row
       const int nrows = (int)imax64(0, imin64(32, ti.row_end - rbase));
       const int64_t grow = rbase + lane;
       const bool vrow = lane < nrows;
@@ -853,12 +837,10 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
           const int blk = hb >> 1, half = hb & 1;
           const int64_t cb = n0 + blk * 128;
           if (cb >= p.N) break;
-          if (hsel >= 0 && (blk * 128) / (BN / 2) != hsel) continue;  // the other column half
-          const int tblk = blk * 128 - (hsel > 0 ? BN / 2 : 0);        // its TMEM columns
           {
             float u[32], a[32];
-            tmem_ld32(tbase + tblk + half * 32, v);
-            tmem_ld32(tbase + tblk + 64 + half * 32, u);
+            tmem_ld32(tbase + blk * 128 + half * 32, v);
+            tmem_ld32(tbase + blk * 128 + 64 + half * 32, u);
 #pragma unroll
             for (int i = 0; i < 32; ++i) a[i] = silu_f(v[i]) * u[i];
 #pragma unroll
@@ -910,8 +892,7 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
         for (int c = ch; c < BN / 32; c += CSTEP) {
           const int64_t col0 = n0 + c * 32;
           if (col0 >= p.N) break;
-          if (hsel >= 0 && (c * 32) / (BN / 2) != hsel) continue;  // the other column half
-          tmem_ld32(tbase + c * 32 - (hsel > 0 ? BN / 2 : 0), v);
+          tmem_ld32(tbase + c * 32, v);
           const int nvalid = (int)imin64(32, p.N - col0);
           if (EPI == 1 || nvalid < 32) {
             // router logits (E columns, possibly ragged): direct row stores
