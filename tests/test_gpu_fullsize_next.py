@@ -1,0 +1,80 @@
+"""Full-size parity of the next-step rows at the base workload (T=8192, D=2048,
+E=64, K=6, F=1024), in the launch configuration bench.py times for them:
+the sigmoid router (``--router sigmoid``) and the shared expert
+(``--shared-width 2688``).  Index work on every token, statistics and router
+gradients over all tokens, the shared expert on sampled tokens and its whole
+weight gradients; tolerances as in the other parity tests."""
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+import synth
+from tests.gpu_util import REL_FROB, f64, i64, rel_frob
+
+pytestmark = pytest.mark.gpu
+
+W = synth.get("C2")
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    import __graft_entry__
+    __graft_entry__.build()
+
+
+def _w64(t):
+    return t.detach().to(torch.float64).numpy()
+
+
+def test_sigmoid_router_full_size():
+    from paper_2608_28511_gb300.layer import MoeLayer
+    inp = synth.make_inputs(W)
+    inp["expert_bias"] = synth.make_expert_bias(W.E, W.seed)
+    L = MoeLayer(W.S, W.GBS, W.K, W.D, W.E, W.F, W.dtype, W.H, router="sigmoid")
+    L.load(inp)
+    L.forward()
+    L.backward()
+    torch.cuda.synchronize()
+    z = f64(L.logits)
+    bias = inp["expert_bias"].double().numpy()
+    idx_ref, _ = O.sigmoid_route(z, W.K, bias)
+    idx = i64(L.topk_idx)
+    keys = O.sigmoid(z) + bias[None, :]
+    top = -np.sort(-keys, axis=1)[:, : W.K + 1]
+    ties = set(np.nonzero((top[:, :-1] - top[:, 1:] < 1e-6).any(axis=1))[0].tolist())
+    differ = set(np.nonzero((idx != idx_ref).any(axis=1))[0].tolist())
+    assert differ <= ties
+    _, prob_at = O.sigmoid_route(z, W.K, bias, idx_override=idx)
+    assert np.abs(f64(L.topk_prob) - prob_at).max() <= 1e-5
+    loss_ref, f_ref, _ = O.seq_aux_loss(z, idx, W.S, W.GBS, L.aux_coef)
+    assert np.array_equal(f64(L.aux_f), f_ref.astype(np.float32).astype(np.float64))
+    assert abs(float(L.aux_loss[0].item()) - loss_ref) <= 1e-4 * abs(loss_ref)
+    dz_ref, _, dw_ref = O.sigmoid_route_bwd(_w64(inp["x"]), _w64(inp["w_router"]), z, idx, f64(L.topk_prob),
+                                            f64(L.dprob), f64(L.aux_f), W.S, W.GBS, L.aux_coef, 1.0)
+    assert rel_frob(f64(L.dlogits), dz_ref) <= 1e-4
+    assert rel_frob(f64(L.dw_router), dw_ref) <= REL_FROB
+
+
+def test_shared_expert_full_size():
+    from paper_2608_28511_gb300.layer import MoeLayer
+    Fs = 2688
+    inp = synth.make_inputs(W)
+    inp.update(synth.make_shared_expert(W, Fs, W.seed))
+    L = MoeLayer(W.S, W.GBS, W.K, W.D, W.E, W.F, W.dtype, W.H, shared_F=Fs)
+    L.load(inp)
+    L.forward()
+    L.backward()
+    torch.cuda.synchronize()
+    x, w1, w2, dy = (_w64(inp[k]) for k in ("x", "w_s1", "w_s2", "dy"))
+    # sampled tokens: the shared expert's pre-activation, activation and its part of y
+    rng = np.random.default_rng(7)
+    toks = np.unique(np.concatenate([[0, W.T - 1], rng.choice(W.T, 48, replace=False)]))
+    h_ref, a_ref, y_ref = O.shared_expert(x[toks], w1, w2)
+    assert rel_frob(f64(L.h_s)[toks], h_ref) <= REL_FROB
+    assert rel_frob(f64(L.act_s)[toks], a_ref) <= REL_FROB
+    # whole weight gradients from the GPU's saved h and act (stage-isolated)
+    dh_ref, _, dw1_ref, dw2_ref = O.shared_expert_bwd(dy, x, f64(L.h_s), f64(L.act_s), w1, w2)
+    assert rel_frob(f64(L.dw_s1), dw1_ref) <= REL_FROB
+    assert rel_frob(f64(L.dw_s2), dw2_ref) <= REL_FROB
+    assert rel_frob(f64(L.dh_s)[toks], dh_ref[toks]) <= REL_FROB
