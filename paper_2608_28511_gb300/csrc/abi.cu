@@ -606,8 +606,10 @@ static int expert_ffn_bwd_impl(const Ctx& c, const Dims& d, const void* dy_perm,
     TRY_CUDA(launch_swiglu_bwd(c, d.dt, dA, h_save, d.TK, d.F, dH));
   }
   TRY_CUDA(gemm(c, b, "ffn2_wgrad_tc", "ffn2_wgrad_simt"));
-  if (d.TK > 0) TRY_CUDA(gemm(c, cg, "ffn1_dgrad_tc", "ffn1_dgrad_simt"));
   TRY_CUDA(gemm(c, w, "ffn1_wgrad_tc", "ffn1_wgrad_simt"));
+  // dgrad-1 last: the dispatch backward that follows reads its output while
+  // part of it is still in L2 (the weight gradients' fp32 writes would flush it)
+  if (d.TK > 0) TRY_CUDA(gemm(c, cg, "ffn1_dgrad_tc", "ffn1_dgrad_simt"));
   return MOE_OK;
 }
 
