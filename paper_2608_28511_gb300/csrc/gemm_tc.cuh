@@ -72,7 +72,7 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
   if (CL)
     asm volatile(
         "{\n\t.reg .pred p;\n\t"
-        "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
         "selp.u32 %0, 1, 0, p;\n\t}\n"
         : "=r"(ok)
         : "r"(bar), "r"(parity)
@@ -180,7 +180,7 @@ __device__ __forceinline__ uint32_t map_to_rank(uint32_t saddr, uint32_t rank) {
   return r;
 }
 __device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
-  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
+  asm volatile("mbarrier.arrive.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
 }
 __device__ __forceinline__ void cluster_sync() {
   asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
@@ -260,9 +260,10 @@ __device__ __forceinline__ void mma_commit_cg(uint32_t bar, uint16_t mask) {
     mma_commit(bar);
 }
 
-// 32 consecutive fp32 columns of this warp's 32 TMEM lanes (one row per thread).
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
-  uint32_t r[32];
+// 32 consecutive fp32 columns of this warp's 32 TMEM lanes (one row per
+// thread), issued without waiting: the registers hold the values only after
+// tmem_ld_wait(r), which every use must follow.
+__device__ __forceinline__ void tmem_ld32_issue(uint32_t taddr, uint32_t (&r)[32]) {
   asm volatile(
       "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
       "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
@@ -271,8 +272,12 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
         "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
         "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
         "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
-      : "r"(taddr));
-  // the registers are tied to the wait so no use is scheduled before it
+      : "r"(taddr)
+      : "memory");
+}
+// Waits for every tcgen05.ld this thread issued; the registers of r are tied
+// to the wait so that no use of them is scheduled before it.
+__device__ __forceinline__ void tmem_ld_wait(uint32_t (&r)[32]) {
   asm volatile("tcgen05.wait::ld.sync.aligned;"
                : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]), "+r"(r[7]),
                  "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]), "+r"(r[14]),
@@ -281,6 +286,11 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
                  "+r"(r[29]), "+r"(r[30]), "+r"(r[31])
                :
                : "memory");
+}
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
+  uint32_t r[32];
+  tmem_ld32_issue(taddr, r);
+  tmem_ld_wait(r);
 #pragma unroll
   for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
@@ -886,6 +896,32 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
             __syncwarp();
             stage_store<RB>(stg, lane, c_rows + col0 * sizeof(TC), ldc_b, nrows);
           }
+        }
+      } else if (EPI == 0 && n0 + BN <= p.N) {
+        // every column of the tile exists: chunk i + 1's TMEM load is in
+        // flight while chunk i is staged and stored
+        constexpr int NC = BN / 32 / CSTEP;  // this warp's chunks: ch, ch + CSTEP, ...
+        static_assert(RPC == 1 && NC % 2 == 0, "one staging round per chunk, chunks in pairs");
+        uint32_t ra[32], rb[32];
+        auto put = [&](const uint32_t(&r)[32], int i) {
+#pragma unroll
+          for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
+#pragma unroll
+          for (int j = 0; j < NP; ++j) pk[j] = pack16<TC>(v + j * Vec<TC>::N);
+          __syncwarp();
+          stage_put<RB>(stg, lane, pk);
+          __syncwarp();
+          stage_store<RB>(stg, lane, c_rows + (n0 + (ch + i * CSTEP) * 32) * sizeof(TC), ldc_b, nrows);
+        };
+        tmem_ld32_issue(tbase + ch * 32, ra);
+#pragma unroll 1
+        for (int i = 0; i < NC; i += 2) {
+          tmem_ld_wait(ra);
+          tmem_ld32_issue(tbase + (ch + (i + 1) * CSTEP) * 32, rb);
+          put(ra, i);
+          tmem_ld_wait(rb);
+          if (i + 2 < NC) tmem_ld32_issue(tbase + (ch + (i + 2) * CSTEP) * 32, ra);
+          put(rb, i + 1);
         }
       } else {
 #pragma unroll 1
