@@ -209,6 +209,89 @@ class MoeLayer:
         return g
 
     # ------------------------------------------------------------------
+    # Steps on batches in pinned host memory, copies overlapped with compute
+    _IO = ("x", "dy", "y", "dx")
+
+    def _bind(self, bufs: dict) -> None:
+        for k in self._IO:
+            setattr(self, k, bufs[k])
+
+    def prepare_host_pipeline(self, graphs: bool = True) -> None:
+        """Allocate a second set of the step's host-facing buffers (x, dy, y,
+        dx) and, with ``graphs``, capture one CUDA graph per set (each after one
+        eager step).  Called once, before ``run_host``; ``x`` and ``dy`` keep
+        the values they hold."""
+        first = {k: getattr(self, k) for k in self._IO}
+        second = {k: torch.empty_like(v) for k, v in first.items()}
+        second["x"].copy_(first["x"])
+        second["dy"].copy_(first["dy"])
+        self._sets = [first, second]
+        self._graphs = None
+        if graphs:
+            self._graphs = []
+            for bufs in self._sets:
+                self._bind(bufs)
+                self.step()
+                self._graphs.append(self.capture())
+        self._bind(first)
+        self._h2d = torch.cuda.Stream(device=self.x.device)
+        self._d2h = torch.cuda.Stream(device=self.x.device)
+        torch.cuda.synchronize(self.x.device)
+
+    def run_host(self, batches) -> None:
+        """One forward + backward step per batch ``(x, dy, y, dx)`` of pinned
+        host tensors: x and dy are the step's inputs, y and dx receive its
+        outputs.  Step i + 1's inputs are copied in on one copy stream while
+        step i computes, and step i's outputs are copied out on another while
+        step i + 1 computes, the two device buffer sets alternating.  Every
+        copy is ordered after the work already on the current stream, and the
+        current stream waits for the last output copy before this returns
+        (asynchronously: synchronise the stream before reading y and dx)."""
+        if not hasattr(self, "_sets"):
+            raise RuntimeError("call prepare_host_pipeline() first")
+        batches = list(batches)
+        n = len(batches)
+        cs = torch.cuda.current_stream(self.x.device)
+        h2d, d2h = self._h2d, self._d2h
+        ready = [torch.cuda.Event(), torch.cuda.Event()]     # a set's inputs are on the device
+        done = [torch.cuda.Event(), torch.cuda.Event()]      # a set's step finished
+        drained = [torch.cuda.Event(), torch.cuda.Event()]   # a set's outputs are on the host
+        h2d.wait_stream(cs)
+
+        def load(i):
+            b, bufs = i % 2, self._sets[i % 2]
+            with torch.cuda.stream(h2d):
+                if i >= 2:
+                    h2d.wait_event(done[b])                  # step i - 2 no longer reads this set
+                bufs["x"].copy_(batches[i][0], non_blocking=True)
+                bufs["dy"].copy_(batches[i][1], non_blocking=True)
+                ready[b].record(h2d)
+
+        if n:
+            load(0)
+        for i in range(n):
+            b, bufs = i % 2, self._sets[i % 2]
+            if i + 1 < n:
+                load(i + 1)
+            cs.wait_event(ready[b])
+            if i >= 2:
+                cs.wait_event(drained[b])                    # step i - 2's outputs have left this set
+            if self._graphs is not None:
+                self._graphs[b].replay()
+            else:
+                self._bind(bufs)
+                self.step()
+            done[b].record(cs)
+            with torch.cuda.stream(d2h):
+                d2h.wait_event(done[b])
+                batches[i][2].copy_(bufs["y"], non_blocking=True)
+                batches[i][3].copy_(bufs["dx"], non_blocking=True)
+                drained[b].record(d2h)
+        cs.wait_stream(d2h)
+        cs.wait_stream(h2d)
+        self._bind(self._sets[0])
+
+    # ------------------------------------------------------------------
     def unpack_w1_like(self, t: torch.Tensor):
         """Split a packed [E, 2F, D] tensor (w1 or dw1) into gate and up [E, F, D]."""
         v = t.view(self.E, self.F // 64, 2, 64, self.D)
