@@ -1,7 +1,10 @@
 // Host side of the tcgen05 engine: which GemmDesc shapes it takes, tensor-map
 // encoding (cuTensorMapEncodeTiled through the runtime's driver entry point)
 // and the launch of the matching kernel instantiation.
+#include <array>
 #include <cstring>
+#include <map>
+#include <memory>
 #include <mutex>
 
 #include "gemm_tc.cuh"
@@ -48,6 +51,29 @@ bool make_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer, 
 }
 
 bool al16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+
+// Group::K tail templates, one per row count r = 1 .. BK - 1, for MN-major A
+// (and B unless B is gathered) with {64, 64} boxes.  They depend only on the
+// operands' row length and stride (the device replaces the base address), so
+// each combination is encoded once and kept for the life of the process.
+const tc::TailTemplates* tail_templates(const void* a, int64_t a_inner, int64_t a_stride, const void* b,
+                                        int64_t b_inner, int64_t b_stride) {
+  static std::mutex mu;
+  static std::map<std::array<int64_t, 5>, std::unique_ptr<tc::TailTemplates>> cache;
+  const std::array<int64_t, 5> key = {a_inner, a_stride, b ? b_inner : -1, b ? b_stride : -1, 0};
+  std::lock_guard<std::mutex> lk(mu);
+  auto it = cache.find(key);
+  if (it != cache.end()) return it->second.get();
+  auto t = std::make_unique<tc::TailTemplates>();
+  memset(t.get(), 0, sizeof(tc::TailTemplates));
+  for (int r = 1; r < tc::BK; ++r) {
+    if (!make_map(&t->a[r], a, a_inner, r, a_stride, 64, 64)) return nullptr;
+    if (b && !make_map(&t->b[r], b, b_inner, r, b_stride, 64, 64)) return nullptr;
+  }
+  const tc::TailTemplates* out = t.get();
+  cache.emplace(key, std::move(t));
+  return out;
+}
 
 struct Plan {
   int bn;
@@ -239,14 +265,16 @@ cudaError_t launch_gemm_tc(const Ctx& c, const GemmDesc& d, const char* name) {
   if (ub <= 0) return cudaSuccess;
   const int g = (int)d.group, e = (int)d.epi;
   if (d.group == Group::K) {
-    // per-group maps: the templates above with the base and row extent moved per group
+    // tail maps: host-encoded templates of 1 .. BK - 1 rows, the base moved per group
+    const tc::TailTemplates* tails = tail_templates(d.A, a_inner, pl.lda * 2, gb ? nullptr : d.B, b_inner, pl.ldb * 2);
+    if (!tails) return cudaErrorInvalidValue;
     CUtensorMap* maps = static_cast<CUtensorMap*>(d.scratch);
     int32_t* split_offs = d.offsets ? nullptr : reinterpret_cast<int32_t*>(maps + 2 * d.num_groups);
     {
       KernelScope ks("group_maps", c.stream);
-      tc::build_group_maps<<<(d.num_groups + 127) / 128, 128, 0, c.stream>>>(
-          p.ta, p.tb, d.offsets, d.num_groups, d.split_rows, split_offs, static_cast<const uint8_t*>(d.A),
-          pl.lda * 2, gb ? nullptr : static_cast<const uint8_t*>(d.B), pl.ldb * 2, maps);
+      tc::build_group_maps<<<(d.num_groups + tc::kMapWarps - 1) / tc::kMapWarps, 32 * tc::kMapWarps, 0, c.stream>>>(
+          *tails, d.offsets, d.num_groups, d.split_rows, split_offs, static_cast<const uint8_t*>(d.A), pl.lda * 2,
+          gb ? nullptr : static_cast<const uint8_t*>(d.B), pl.ldb * 2, maps);
     }
     cudaError_t st = cudaGetLastError();
     if (st != cudaSuccess) return st;

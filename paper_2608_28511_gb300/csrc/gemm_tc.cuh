@@ -46,7 +46,7 @@ struct Params {
   const float* bias;
   void* aux;
   uint32_t* err;
-  const CUtensorMap* gmaps;  // Group::K: per group {A, B} maps whose rows start at the group's first row
+  const CUtensorMap* gmaps;  // Group::K: per group {A, B} maps of its last rows (fewer than BK)
   const int32_t* gather;     // GATHER: source row of each gathered row (the permutation's token_of_row)
 };
 
@@ -571,7 +571,6 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
     uint32_t phase = 0;
     int issued = 0;
     uint32_t last_phase = 0;
-    int cur_g = -1;
     bool ok = true;
     for (int t = cta0; t < total && ok; t += ncta) {
       Tile ti;
@@ -618,17 +617,19 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
             }
           }
         } else {
-          // A from the group's own map (zero past the group's rows); B's 64 k
-          // rows from the source, in 64-column chunks of 16 four-row copies
+          // A: whole k-blocks from the full map, the group's last rows from
+          // its tail map (zero past the group's rows); B's 64 k rows from the
+          // source, in 64-column chunks of 16 four-row copies
           if (lane == 0) {
-            const CUtensorMap* ma = p.gmaps + 2 * ti.g;
-            if (ti.g != cur_g) {
+            if (kb < (int)((ti.kend - ti.kbeg) / BK)) {
+              load(sa, &p.ta, (int)ti.row0, k0);
+              load(sa + 8192, &p.ta, (int)ti.row0 + 64, k0);
+            } else {
+              const CUtensorMap* ma = p.gmaps + 2 * ti.g;
               tmap_acquire(ma);
-              cur_g = ti.g;
+              load(sa, ma, (int)ti.row0, 0);
+              load(sa + 8192, ma, (int)ti.row0 + 64, 0);
             }
-            const int ky = kb * BK;
-            load(sa, ma, (int)ti.row0, ky);
-            load(sa + 8192, ma, (int)ti.row0 + 64, ky);
           }
 #pragma unroll
           for (int u = lane; u < (BNC / 64) * 16; u += 32) {
@@ -648,6 +649,19 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
         if (++stage == C::kStages) { stage = 0; phase ^= 1u; }
       }
     }
+    // tail: wait until the MMA warp has released every stage this CTA filled.
+    // Its releases are asynchronous arrivals (multicast to both CTAs of a pair)
+    // that may still be in flight when the MMAs are done; waiting here keeps
+    // either CTA from exiting before they land in its shared memory.  Stages
+    // never filled pass at once.
+    if (lane == 0 && ok) {
+      int s = stage;
+      uint32_t ph = phase;
+      for (int i = 0; i < C::kStages; ++i) {
+        wait_drain<CG == 2>(smem_u32(&empty[s]), ph ^ 1u, 1000000000ull);
+        if (++s == C::kStages) { s = 0; ph ^= 1u; }
+      }
+    }
     if (leader && lane == 0) {
       const int pending = issued < C::kStages ? issued : C::kStages;
       for (int i = 0; i < pending; ++i) {
@@ -662,7 +676,6 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
       uint32_t phase = 0;
       int issued = 0;
       uint32_t last_phase = 0;  // bit s: phase of the last copy issued into stage s
-      int cur_g = -1;           // group whose maps this thread has acquired (Group::K)
       bool ok = true;
       for (int t = cta0; t < total && ok; t += ncta) {
         Tile ti;
@@ -682,17 +695,20 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
             else tma_load_2d(dst, m, fb, x, y);
           };
           if (GROUP == 2) {
-            // the group's own maps: k rows count from the group's first row and
-            // the copy engine zero-fills rows past its end (the next group's rows
-            // never enter the reduction)
-            const CUtensorMap* ma = p.gmaps + 2 * ti.g;
-            const CUtensorMap* mb = ma + 1;
-            if (ti.g != cur_g) {
+            // whole k-blocks of the group from the full-tensor maps at absolute
+            // rows; its last n % BK rows from the group's tail maps, whose row
+            // extent ends at the group's end, so the copy engine zero-fills the
+            // rest of the block (the next group's rows never enter the reduction)
+            const CUtensorMap* ma = &p.ta;
+            const CUtensorMap* mb = &p.tb;
+            int ky = k0;
+            if (kb >= (int)((ti.kend - ti.kbeg) / BK)) {
+              ma = p.gmaps + 2 * ti.g;
+              mb = ma + 1;
               tmap_acquire(ma);
               tmap_acquire(mb);
-              cur_g = ti.g;
+              ky = 0;
             }
-            const int ky = kb * BK;
             load(sa, ma, (int)ti.row0, ky);
             load(sa + 8192, ma, (int)ti.row0 + 64, ky);
 #pragma unroll
@@ -715,6 +731,16 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
           last_phase = (last_phase & ~(1u << stage)) | (phase << stage);
           ++issued;
           if (++stage == C::kStages) { stage = 0; phase ^= 1u; }
+        }
+      }
+      // tail: wait until the MMA warp has released every stage this CTA
+      // filled (see the gathering producer above)
+      if (ok) {
+        int s = stage;
+        uint32_t ph = phase;
+        for (int i = 0; i < C::kStages; ++i) {
+          wait_drain<CG == 2>(smem_u32(&empty[s]), ph ^ 1u, 1000000000ull);
+          if (++s == C::kStages) { s = 0; ph ^= 1u; }
         }
       }
       // drain: every issued copy must land before the CTA exits (the leader's
@@ -996,18 +1022,35 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
   if (warp == 1) tmem_dealloc_cg<CG>(tmem_base, C::kCols);
 }
 
-// Per-group tensor maps for Group::K: group g's A and B maps are copies of
-// the full-tensor templates with the base moved to the group's first row and
-// the row extent set to the group's row count (at least 1), so a copy that
-// runs past the group's rows reads zeros.  out[2g] = A, out[2g + 1] = B.
-// With offsets == nullptr the groups are G equal splits of [0, split_rows)
-// and their offsets are written to offs_out for the GEMM to read.
-__global__ void build_group_maps(const __grid_constant__ CUtensorMap ta, const __grid_constant__ CUtensorMap tb,
-                                 const int32_t* __restrict__ offsets, int G, int64_t split_rows,
-                                 int32_t* __restrict__ offs_out, const uint8_t* a_base, int64_t a_row_bytes,
-                                 const uint8_t* b_base, int64_t b_row_bytes, CUtensorMap* out) {
-  const int g = blockIdx.x * blockDim.x + threadIdx.x;
-  if (g >= G) return;
+// Tail maps for Group::K.  A group's whole k-blocks are read through the
+// full-tensor maps; its last r = n % BK rows (0 < r < BK) through tail maps:
+// host-encoded templates of exactly r rows (TailTemplates, one per r) whose
+// base the device moves to the group's first tail row.  Only the address is
+// replaced on the device, which leaves a map identical to a host encoding of
+// the same tensor; the copy engine zero-fills the block's rows past the
+// group's end, so the next group's rows never enter the reduction, and every
+// map's base lies inside its tensor.  out[2g] = A, out[2g + 1] = B (none for
+// a group whose row count is a multiple of BK).  With offsets == nullptr the
+// groups are G equal splits of [0, split_rows) and their offsets are written
+// to offs_out for the GEMM to read.
+// One warp per group: the template is copied into shared memory, its address
+// is replaced there (tensormap.replace on shared::cta), and the warp copies
+// the finished map to global memory with tensormap.cp_fenceproxy, which
+// releases it to the tensormap proxy; the GEMM's producer acquires it before
+// its copy.
+struct TailTemplates {
+  CUtensorMap a[BK];  // [r]: r rows (r = 1 .. BK - 1)
+  CUtensorMap b[BK];
+};
+constexpr int kMapWarps = 4;
+__global__ void __launch_bounds__(32 * kMapWarps) build_group_maps(
+    const __grid_constant__ TailTemplates tt, const int32_t* __restrict__ offsets, int G, int64_t split_rows,
+    int32_t* __restrict__ offs_out, const uint8_t* a_base, int64_t a_row_bytes, const uint8_t* b_base,
+    int64_t b_row_bytes, CUtensorMap* out) {
+  __shared__ alignas(128) CUtensorMap sm[kMapWarps][2];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int g = blockIdx.x * kMapWarps + warp;
+  if (g >= G) return;  // the whole warp
   int64_t lo, hi;
   if (offsets) {
     lo = offsets[g];
@@ -1015,30 +1058,42 @@ __global__ void build_group_maps(const __grid_constant__ CUtensorMap ta, const _
   } else {
     lo = split_rows * g / G;
     hi = split_rows * (g + 1) / G;
-    offs_out[g] = (int32_t)lo;
-    if (g == G - 1) offs_out[G] = (int32_t)hi;
+    if (lane == 0) {
+      offs_out[g] = (int32_t)lo;
+      if (g == G - 1) offs_out[G] = (int32_t)hi;
+    }
   }
-  const int64_t rows = hi - lo;
-  const uint32_t dim = rows > 0 ? (uint32_t)rows : 1u;
-  CUtensorMap* ma = out + 2 * g;
-  CUtensorMap* mb = ma + 1;
-  const uint4* sa = reinterpret_cast<const uint4*>(&ta);
-  const uint4* sb = reinterpret_cast<const uint4*>(&tb);
-  uint4* da = reinterpret_cast<uint4*>(ma);
-  uint4* db = reinterpret_cast<uint4*>(mb);
-#pragma unroll
-  for (int i = 0; i < 8; ++i) da[i] = sa[i];
-  const uint64_t pa = reinterpret_cast<uint64_t>(a_base + lo * a_row_bytes);
-  asm volatile("tensormap.replace.tile.global_address.global.b1024.b64 [%0], %1;" ::"l"(ma), "l"(pa) : "memory");
-  asm volatile("tensormap.replace.tile.global_dim.global.b1024.b32 [%0], 1, %1;" ::"l"(ma), "r"(dim) : "memory");
-  if (b_base) {  // NULL: B is gathered through one full map (no per-group B map)
-#pragma unroll
-    for (int i = 0; i < 8; ++i) db[i] = sb[i];
-    const uint64_t pb = reinterpret_cast<uint64_t>(b_base + lo * b_row_bytes);
-    asm volatile("tensormap.replace.tile.global_address.global.b1024.b64 [%0], %1;" ::"l"(mb), "l"(pb) : "memory");
-    asm volatile("tensormap.replace.tile.global_dim.global.b1024.b32 [%0], 1, %1;" ::"l"(mb), "r"(dim) : "memory");
+  const int r = (int)((hi - lo) % BK);
+  if (r == 0) return;  // no tail: every k-block of the group is whole
+  const int64_t first = hi - r;
+  const bool has_b = b_base != nullptr;  // NULL: B is gathered through one full map (no tail B map)
+  // 32 lanes x 4 bytes = one 128-byte map
+  reinterpret_cast<uint32_t*>(&sm[warp][0])[lane] = reinterpret_cast<const uint32_t*>(&tt.a[r])[lane];
+  if (has_b) reinterpret_cast<uint32_t*>(&sm[warp][1])[lane] = reinterpret_cast<const uint32_t*>(&tt.b[r])[lane];
+  __syncwarp();
+  const uint32_t sa = smem_u32(&sm[warp][0]), sb = smem_u32(&sm[warp][1]);
+  if (lane == 0) {
+    const uint64_t pa = reinterpret_cast<uint64_t>(a_base + first * a_row_bytes);
+    asm volatile("tensormap.replace.tile.global_address.shared::cta.b1024.b64 [%0], %1;" ::"r"(sa), "l"(pa)
+                 : "memory");
+    if (has_b) {
+      const uint64_t pb = reinterpret_cast<uint64_t>(b_base + first * b_row_bytes);
+      asm volatile("tensormap.replace.tile.global_address.shared::cta.b1024.b64 [%0], %1;" ::"r"(sb), "l"(pb)
+                   : "memory");
+    }
   }
-  asm volatile("fence.proxy.tensormap::generic.release.gpu;" ::: "memory");
+  __syncwarp();
+  asm volatile(
+      "tensormap.cp_fenceproxy.global.shared::cta.tensormap::generic.release.gpu.sync.aligned [%0], [%1], 128;" ::"l"(
+          reinterpret_cast<uint64_t>(out + 2 * g)),
+      "r"(sa)
+      : "memory");
+  if (has_b)
+    asm volatile(
+        "tensormap.cp_fenceproxy.global.shared::cta.tensormap::generic.release.gpu.sync.aligned [%0], [%1], 128;" ::
+            "l"(reinterpret_cast<uint64_t>(out + 2 * g + 1)),
+        "r"(sb)
+        : "memory");
 }
 
 }  // namespace tc
