@@ -74,6 +74,8 @@ def kernel_work(name: str, w: synth.Workload, T: int, Fs: int = 0) -> tuple[str,
         "route_dz_sigmoid": T * E * 4 + T * K * 12 + T * E * 6,
         "swiglu_bwd": 5.0 * TK * F * bx,
         "relusq_bwd": 3.0 * T * Fs * bx,
+        "dispatch_fp8": T * D * bx + TK * D + 8 * TK,
+        "dequant_rows": TK * D + TK * D * bx + 4 * TK,
         "pack_w1": 0.0,
     }
     return "hbm", float(byts.get(base, 0.0))
@@ -263,6 +265,8 @@ def main() -> None:
     ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--no-graph", action="store_true",
                     help="launch every kernel from the host each step instead of replaying a captured CUDA graph")
+    ap.add_argument("--payload", default="bf16", choices=["bf16", "fp8"],
+                    help="dispatch payload: bf16 rows, or FP8 E4M3 codes with a power-of-two scale per row")
     ap.add_argument("--shared-width", type=int, default=0,
                     help="hidden units of the ungated shared expert (0 = none; Sec. 5.2)")
     ap.add_argument("--router", default="softmax", choices=["softmax", "sigmoid"],
@@ -296,7 +300,8 @@ def main() -> None:
         inputs["expert_bias"] = synth.make_expert_bias(w.E, rank_seed(w, rank))
     if args.shared_width:
         inputs.update(synth.make_shared_expert(w, args.shared_width, rank_seed(w, rank)))
-    L = MoeLayer(w.S, w.GBS, w.K, w.D, w.E, w.F, w.dtype, w.H, router=args.router, shared_F=args.shared_width)
+    L = MoeLayer(w.S, w.GBS, w.K, w.D, w.E, w.F, w.dtype, w.H, router=args.router, shared_F=args.shared_width,
+                 payload=args.payload)
     L.load(inputs)
     stream = torch.cuda.current_stream()
     flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device="cuda")
@@ -426,7 +431,8 @@ def main() -> None:
               for k, v in sorted(kernels.items(), key=lambda kv: -kv[1]["ms_per_step"])}
 
     cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline and args.router == "softmax" and not args.shared_width:
+    if (rank == 0 and world == 1 and not args.no_cpu_baseline and args.router == "softmax" and not args.shared_width
+            and args.payload == "bf16"):
         cpu = cpu_baseline(w, args.cpu_budget)
 
     if rank == 0:
@@ -436,6 +442,7 @@ def main() -> None:
             "scaling": "weak", "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
             "config": {"workload": w.name, "T": T, "S": w.S, "GBS": w.GBS, "D": w.D, "E": w.E, "K": w.K, "F": w.F,
                        "H": w.H, "seed": w.seed, "router": args.router, "shared_width": args.shared_width,
+                       "payload": args.payload,
                        "parallelism": f"replicas x{world}, each rank its own tokens",
                        "launch": "one CUDA graph per step" if graph is not None else "eager launches",
                        "l2": "256 MiB buffer written before every timed step (outside the step events); "

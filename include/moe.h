@@ -114,6 +114,24 @@ int moe_dispatch(const moe_shape_t* shape, const void* x, const int32_t* topk_id
                  int32_t* expert_offsets, int32_t* row_of_slot, int32_t* token_of_row,
                  void* x_perm, float* prob_perm, void* ws, size_t ws_bytes, void* stream);
 
+/* Dispatch with a low-precision payload (Sec. 1: lower-precision
+ * communication, b_x of Eq. 1; readings FP1-FP2): the permutation and
+ * prob_perm as moe_dispatch, and each token's row of x [T, D] (bf16 only;
+ * MOE_ERR_UNSUPPORTED otherwise) sent to its K rows as FP8 E4M3 codes,
+ * x_perm_q [TK, D] (one byte each), with one fp32 scale per row,
+ * x_scale_perm [TK]: the smallest power of two s = 2^e, e >= -126, with
+ * max_i |x_i| <= 448 s (1 for an all-zero row); code_i = the E4M3 value nearest
+ * x_i / s, ties to even, saturating at +-448.  The payload per routed slot is
+ * D + 4 + 4 bytes (codes, scale, probability) instead of 2 D + 4. */
+int moe_dispatch_fp8(const moe_shape_t* shape, const void* x, const int32_t* topk_idx, const float* topk_prob,
+                     int32_t* expert_offsets, int32_t* row_of_slot, int32_t* token_of_row, void* x_perm_q,
+                     float* x_scale_perm, float* prob_perm, void* ws, size_t ws_bytes, void* stream);
+
+/* The receiving side of moe_dispatch_fp8: x_perm[r, i] = value(code) * scale[r]
+ * in bf16 ([TK, D]; exact, the scale being a power of two). */
+int moe_dequant_rows(const moe_shape_t* shape, const void* x_perm_q, const float* x_scale_perm, void* x_perm,
+                     void* stream);
+
 /* Dispatch that allocates nothing and takes no workspace.  The paper has no
  * counterpart: this entry point exists for callers that cannot allocate
  * device memory when they call the layer -- a host framework that has already

@@ -91,6 +91,12 @@ cudaError_t launch_dispatch_bwd(const Ctx& c, DType dt, const void* dx_perm, con
 cudaError_t launch_pack_w1(const Ctx& c, DType dt, const void* w_gate, const void* w_up, int E, int F, int D,
                            void* w1);
 
+// fp8_payload.cu: E4M3 codes [TK, D] and power-of-two row scales [TK] of the
+// bf16 rows x [T, D] written to each token's K rows; and their bf16 values.
+cudaError_t launch_dispatch_fp8(const Ctx& c, const void* x, const int32_t* row_of_slot, int64_t T, int K, int D,
+                                void* xq, float* scale_perm);
+cudaError_t launch_dequant_rows(const Ctx& c, const void* xq, const float* scale, int64_t rows, int D, void* out);
+
 // swiglu.cu: dH [rows, 2F] (packed) from dA [rows, F] and the saved h [rows, 2F].
 cudaError_t launch_swiglu_bwd(const Ctx& c, DType dt, const void* dA, const void* h, int64_t rows, int F,
                               void* dH);

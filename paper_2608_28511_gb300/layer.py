@@ -32,14 +32,20 @@ class MoeLayer:
     back with tiled copies, which is faster on GB300 (a four-row gather of
     128-byte rows moves far fewer bytes per copy-engine operation than a
     128-row tile).
+    ``payload="fp8"`` dispatches the hidden rows as FP8 E4M3 codes with one
+    power-of-two scale per row (b_x = 1) and dequantizes them on arrival;
+    the gradient passes the quantization unchanged.
     """
 
     def __init__(self, S, GBS, K, D, E, F, dtype="bf16", H=0, device="cuda", router="softmax", aux_coef=1e-4,
-                 aux_grad=1.0, shared_F=0, gather=False):
+                 aux_grad=1.0, shared_F=0, gather=False, payload="bf16"):
         if router not in ("softmax", "sigmoid"):
             raise ValueError(f"unknown router {router!r}")
         self.router = router
         self.gather = bool(gather)
+        if payload not in ("bf16", "fp8") or (payload == "fp8" and (gather or dtype != "bf16")):
+            raise ValueError(f"payload {payload!r} with gather={gather}, dtype={dtype}")
+        self.payload = payload
         self.aux_coef = float(aux_coef)
         self.aux_grad = float(aux_grad)
         self.shape = abi.MoeShape.of(S, GBS, K, D, E, F, dtype, H)
@@ -76,6 +82,8 @@ class MoeLayer:
         self.row_of_slot = e(TK, d=i32)
         self.token_of_row = e(TK, d=i32)
         self.x_perm = None if self.gather else e(TK, D)
+        self.x_perm_q = e(TK, D, d=torch.uint8) if payload == "fp8" else None
+        self.x_scale_perm = e(TK, d=f32) if payload == "fp8" else None
         self.prob_perm = e(TK, d=f32)
         self.h = e(TK, 2 * F)
         self.act = e(TK, F)
@@ -140,8 +148,13 @@ class MoeLayer:
         if self.H:
             abi.moe_latent_proj(s, self.H, self.D, self.x, self.w_down, self.x_lat, self.ws, stream)
             xd = self.x_lat
-        abi.moe_dispatch(s, xd, self.topk_idx, self.topk_prob, self.expert_offsets, self.row_of_slot,
-                         self.token_of_row, self.x_perm, self.prob_perm, self.ws, stream)
+        if self.payload == "fp8":
+            abi.moe_dispatch_fp8(s, xd, self.topk_idx, self.topk_prob, self.expert_offsets, self.row_of_slot,
+                                 self.token_of_row, self.x_perm_q, self.x_scale_perm, self.prob_perm, self.ws, stream)
+            abi.moe_dequant_rows(s, self.x_perm_q, self.x_scale_perm, self.x_perm, stream)
+        else:
+            abi.moe_dispatch(s, xd, self.topk_idx, self.topk_prob, self.expert_offsets, self.row_of_slot,
+                             self.token_of_row, self.x_perm, self.prob_perm, self.ws, stream)
         if self.gather:
             abi.moe_expert_ffn_gather(s, xd, self.token_of_row, self.expert_offsets, self.w1, self.w2, self.h,
                                       self.act, self.y_perm, self.ws, stream)
