@@ -78,3 +78,38 @@ def test_shared_expert_full_size():
     assert rel_frob(f64(L.dw_s1), dw1_ref) <= REL_FROB
     assert rel_frob(f64(L.dw_s2), dw2_ref) <= REL_FROB
     assert rel_frob(f64(L.dh_s)[toks], dh_ref[toks]) <= REL_FROB
+
+
+def test_fp8_payload_full_size():
+    """The FP8 dispatch payload at the base workload (``--payload fp8``): every
+    token's codes and row scale at all K of its rows, bit for bit against the
+    oracle's quantization of the GPU's own dispatch input; the dequantized
+    rows exactly; sampled tokens' layer output within the layer tolerance,
+    from the dequantized rows (readings FP1-FP3)."""
+    from paper_2608_28511_gb300.layer import MoeLayer
+    inp = synth.make_inputs(W)
+    L = MoeLayer(W.S, W.GBS, W.K, W.D, W.E, W.F, W.dtype, W.H, payload="fp8")
+    L.load(inp)
+    L.forward()
+    L.backward()
+    torch.cuda.synchronize()
+    x = _w64(inp["x"])
+    codes, scales = O.fp8_quantize_rows(x)
+    tor = i64(L.token_of_row)
+    assert np.array_equal(L.x_perm_q.cpu().numpy(), codes[tor])
+    assert np.array_equal(f64(L.x_scale_perm), scales[tor])
+    assert np.array_equal(f64(L.x_perm), O.fp8_dequantize_rows(codes, scales)[tor])
+    # sampled tokens' y from the dequantized rows (stage-isolated routing: the GPU's indices)
+    rng = np.random.default_rng(11)
+    toks = np.unique(np.concatenate([[0, W.T - 1], rng.choice(W.T, 48, replace=False)]))
+    x_deq = O.fp8_dequantize_rows(codes[toks], scales[toks])
+    idx = i64(L.topk_idx)[toks]
+    prob = f64(L.topk_prob)[toks]
+    wg, wu, w2 = (_w64(inp[k]) for k in ("w_gate", "w_up", "w2"))
+    y_ref = np.zeros((len(toks), W.D))
+    for i in range(len(toks)):
+        for k in range(W.K):
+            e = idx[i, k]
+            g, u = x_deq[i] @ wg[e].T, x_deq[i] @ wu[e].T
+            y_ref[i] += prob[i, k] * ((O.silu(g) * u) @ w2[e].T)
+    assert rel_frob(f64(L.y)[toks], y_ref) <= REL_FROB
