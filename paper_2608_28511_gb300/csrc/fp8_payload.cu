@@ -13,13 +13,13 @@ namespace moe {
 
 namespace {
 
-constexpr float kE4M3Max = 448.0f;
-
-// Exponent of the row scale for a row maximum amax (finite, >= 0).
+// Exponent of the row scale for a row maximum amax (finite, >= 0): the
+// smallest e with amax <= 448 2^e, where 448 (the largest finite E4M3 value)
+// is 0.875 2^9.
 __device__ __forceinline__ int row_scale_exp(float amax) {
   if (!(amax > 0.f)) return 0;
   int k;
-  const float m = frexpf(amax, &k);  // amax = m 2^k, m in [0.5, 1); 448 = 0.875 2^9
+  const float m = frexpf(amax, &k);  // amax = m 2^k, m in [0.5, 1)
   const int e = k - 9 + (m > 0.875f ? 1 : 0);
   return e < -126 ? -126 : e;
 }

@@ -83,8 +83,13 @@ CEMOE = Workload("cemoe_T16384_D2048_E128_K8_F1536", S=4096, GBS=4, D=2048, E=12
 LATENT = Workload("latent_T16384_H4096_D1024_E256_K8_F768", S=4096, GBS=4, D=1024, E=256, K=8, F=768, H=4096)
 SKEW = Workload("skew_T32768_D2048_E128_K8_F1024", S=8192, GBS=4, D=2048, E=128, K=8, F=1024, skew_bias=True)
 
-WORKLOADS = {w.name: w for w in (TINY, BASE, CEMOE, LATENT, SKEW)}
-ALIASES = {"C1": TINY, "C2": BASE, "C3": CEMOE, "C4": LATENT, "C5": SKEW}
+# The base workload's shape with half the tokens and half the experts (the same
+# ~768 rows per expert): a case for detailed profiler captures, which replay
+# each kernel many times and save and restore device memory around them.
+BASE_HALF = Workload("base_half_T4096_D2048_E32_K6_F1024", S=2048, GBS=2, D=2048, E=32, K=6, F=1024)
+
+WORKLOADS = {w.name: w for w in (TINY, BASE, CEMOE, LATENT, SKEW, BASE_HALF)}
+ALIASES = {"C1": TINY, "C2": BASE, "C3": CEMOE, "C4": LATENT, "C5": SKEW, "C2h": BASE_HALF}
 
 
 def get(name: str) -> Workload:
