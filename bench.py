@@ -63,7 +63,7 @@ def kernel_work(name: str, w: synth.Workload, T: int, Fs: int = 0) -> tuple[str,
     byts = {
         "router_gemm": T * Din * bx + E * Din * bx + T * E * 4,
         "topk": T * E * 4 + T * K * 8,
-        "perm_hist": TK * 4, "perm_scan": 0.0, "perm_rank": TK * 4 * 2 + TK * 4 * 4,
+        "perm_hist": TK * 4, "perm_rank": TK * 4 * 2 + TK * 4 * 4,
         "dispatch_rows": (T + TK) * D * bx + TK * 4,
         "combine": (TK + T) * D * bx + 8 * TK,
         "combine_bwd": (T + 2 * TK) * D * bx + 12 * TK,

@@ -140,12 +140,12 @@ int moe_dequant_rows(const moe_shape_t* shape, const void* x_perm_q, const float
  * synchronisation -- and so cannot provide the workspace moe_dispatch needs.
  *
  * Results are identical to moe_dispatch (same arguments minus ws/ws_bytes).
- * The counting sort's per-chunk histogram and prefix-sum tables,
- * 2 * E * ceil(T*K / 2048) int32 values, live in one fixed device array of
+ * The counting sort's per-chunk histogram table, E * ceil(T*K / 2048)
+ * int32 values, lives in one fixed device array of
  * MOE_DISPATCH_NOALLOC_SCRATCH_INTS int32 (1 MiB) compiled into the library;
  * every GPU that loads the library holds its copy until the process exits.
  * The call makes no cudaMalloc / cudaFree or other allocating call.
- *  - A shape whose tables do not fit (E * ceil(T*K / 2048) > 131072) returns
+ *  - A shape whose table does not fit (E * ceil(T*K / 2048) > 262144) returns
  *    MOE_ERR_TOO_LARGE before anything is enqueued.
  *  - The first call on a device looks up that device's copy of the array
  *    (cudaGetSymbolAddress, with the device current); make that first call

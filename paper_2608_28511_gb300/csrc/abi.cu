@@ -282,7 +282,7 @@ const char* moe_strerror(int status) {
     case MOE_ERR_CUDA: return "CUDA runtime error (see moe_last_cuda_error)";
     case MOE_ERR_DEVICE: return "device status word set (out-of-range expert index or expired bounded wait)";
     case MOE_ERR_UNSUPPORTED: return "unsupported request";
-    case MOE_ERR_TOO_LARGE: return "shape exceeds the fixed scratch of moe_dispatch_noalloc (E * ceil(T*K/2048) > 131072)";
+    case MOE_ERR_TOO_LARGE: return "shape exceeds the fixed scratch of moe_dispatch_noalloc (E * ceil(T*K/2048) > 262144)";
     default: return "unknown status";
   }
 }

@@ -72,8 +72,7 @@ extern "C" int moe_dispatch_noalloc(const moe_shape_t* shape, const void* x, con
   st = scratch_for_device(c.device, &scratch);
   if (st != MOE_OK) return st;
   // Every table entry the kernels read is written earlier in the same call
-  // (the histogram writes all E x chunks counts, the scan all bases), so no
-  // clearing is needed.
+  // (the histogram writes all E x chunks counts), so no clearing is needed.
   st = abi_cuda_status(launch_permutation(c, topk_idx, topk_prob, d.T, d.K, d.E, expert_offsets, row_of_slot,
                                           token_of_row, prob_perm, scratch));
   if (st != MOE_OK) return st;

@@ -15,7 +15,7 @@ constexpr int kSub = kChunk / kRankWarps;
 static inline int64_t num_chunks(int64_t TK) { return (TK + kChunk - 1) / kChunk; }
 
 size_t perm_workspace_bytes(int64_t TK, int E) {
-  return (size_t)2 * (size_t)E * (size_t)num_chunks(TK) * sizeof(int32_t);
+  return (size_t)E * (size_t)num_chunks(TK) * sizeof(int32_t);
 }
 
 // Per-chunk expert histogram (shared-memory counters; counts are order-free,
@@ -36,48 +36,48 @@ __global__ void __launch_bounds__(256) perm_hist_kernel(const int32_t* __restric
   for (int i = threadIdx.x; i < E; i += blockDim.x) counts[(int64_t)i * nchunks + blockIdx.x] = h[i];
 }
 
-// Exclusive prefix sum over the expert-major (expert, chunk) table, one block.
-// base[e * nchunks + c] = first row of expert e's slots from chunk c;
-// offsets[e] = base[e * nchunks], offsets[E] = number of valid slots.
-__global__ void __launch_bounds__(1024) perm_scan_kernel(const int32_t* __restrict__ counts, int E, int nchunks,
-                                                         int32_t* __restrict__ base, int32_t* __restrict__ offsets) {
-  __shared__ int part[1024];
-  const int n = E * nchunks;
-  const int per = (n + 1023) / 1024;
-  const int beg = min(n, threadIdx.x * per), end = min(n, beg + per);
-  int sum = 0;
-  for (int i = beg; i < end; ++i) sum += counts[i];
-  part[threadIdx.x] = sum;
-  __syncthreads();
-  for (int off = 1; off < 1024; off <<= 1) {
-    const int v = threadIdx.x >= off ? part[threadIdx.x - off] : 0;
-    __syncthreads();
-    part[threadIdx.x] += v;
-    __syncthreads();
-  }
-  int run = threadIdx.x ? part[threadIdx.x - 1] : 0;
-  for (int i = beg; i < end; ++i) {
-    base[i] = run;
-    run += counts[i];
-  }
-  __syncthreads();
-  for (int e = threadIdx.x; e < E; e += 1024) offsets[e] = base[(int64_t)e * nchunks];
-  if (threadIdx.x == 0) offsets[E] = part[1023];
-}
-
 // Ranks every slot of one chunk in slot order (= token order within an
 // expert, since a token picks an expert at most once), so the permutation is
-// stable in t and bit-reproducible.  Warp w owns slots [w * kSub, (w+1) * kSub)
-// of the chunk and walks them 32 at a time; lanes that share an expert get
-// consecutive rows by __match_any_sync rank.  Also writes prob_perm.
+// stable in t and bit-reproducible.  Each block first derives its chunk's
+// first row per expert from the whole (expert, chunk) count table: the
+// exclusive scan of the experts' totals plus the expert's counts in the
+// earlier chunks (block 0 also writes the offsets).  Warp w owns slots
+// [w * kSub, (w+1) * kSub) of the chunk and walks them 32 at a time; lanes
+// that share an expert get consecutive rows by __match_any_sync rank.  Also
+// writes prob_perm.
 __global__ void __launch_bounds__(kRankWarps * 32) perm_rank_kernel(
     const int32_t* __restrict__ idx, const float* __restrict__ prob, int64_t TK, int K, int E, int nchunks,
-    const int32_t* __restrict__ base, int32_t* __restrict__ row_of_slot, int32_t* __restrict__ token_of_row,
-    float* __restrict__ prob_perm) {
+    const int32_t* __restrict__ counts, int32_t* __restrict__ offsets, int32_t* __restrict__ row_of_slot,
+    int32_t* __restrict__ token_of_row, float* __restrict__ prob_perm) {
   __shared__ int cnt[kRankWarps * kMaxE];
+  __shared__ int tot[kMaxE + 1];  // expert totals, then their exclusive scan
+  __shared__ int pre[kMaxE];      // the expert's slots in the chunks before this one
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   for (int i = threadIdx.x; i < kRankWarps * E; i += blockDim.x) cnt[i] = 0;
+  for (int e = threadIdx.x; e < E; e += blockDim.x) {
+    const int32_t* row = counts + (int64_t)e * nchunks;
+    int before = 0, all = 0;
+    for (int c = 0; c < nchunks; ++c) {
+      const int v = row[c];
+      before += c < (int)blockIdx.x ? v : 0;
+      all += v;
+    }
+    pre[e] = before;
+    tot[e] = all;
+  }
   __syncthreads();
+  if (threadIdx.x == 0) {  // E <= 256: a serial scan is a few hundred adds
+    int run = 0;
+    for (int e = 0; e < E; ++e) {
+      const int v = tot[e];
+      tot[e] = run;
+      run += v;
+    }
+    tot[E] = run;
+  }
+  __syncthreads();
+  if (blockIdx.x == 0)
+    for (int e = threadIdx.x; e <= E; e += blockDim.x) offsets[e] = tot[e];
   const int64_t c0 = (int64_t)blockIdx.x * kChunk;
   const int64_t w0 = c0 + (int64_t)warp * kSub;
   const int64_t w1 = min(TK, w0 + kSub);
@@ -87,7 +87,7 @@ __global__ void __launch_bounds__(kRankWarps * 32) perm_rank_kernel(
   }
   __syncthreads();
   for (int e = threadIdx.x; e < E; e += blockDim.x) {
-    int run = base[(int64_t)e * nchunks + blockIdx.x];
+    int run = tot[e] + pre[e];
     for (int w = 0; w < kRankWarps; ++w) {
       const int c = cnt[w * E + e];
       cnt[w * E + e] = run;
@@ -124,7 +124,6 @@ cudaError_t launch_permutation(const Ctx& c, const int32_t* idx, const float* pr
   const int64_t TK = T * K;
   const int nch = (int)num_chunks(TK);
   int32_t* counts = (int32_t*)ws;
-  int32_t* base = counts + (int64_t)E * nch;
   if (TK == 0) {
     KernelScope ks("perm_zero", c.stream);
     return cudaMemsetAsync(offsets, 0, sizeof(int32_t) * (E + 1), c.stream);
@@ -136,15 +135,9 @@ cudaError_t launch_permutation(const Ctx& c, const int32_t* idx, const float* pr
   cudaError_t st = cudaGetLastError();
   if (st != cudaSuccess) return st;
   {
-    KernelScope ks("perm_scan", c.stream);
-    perm_scan_kernel<<<1, 1024, 0, c.stream>>>(counts, E, nch, base, offsets);
-  }
-  st = cudaGetLastError();
-  if (st != cudaSuccess) return st;
-  {
     KernelScope ks("perm_rank", c.stream);
-    perm_rank_kernel<<<nch, kRankWarps * 32, 0, c.stream>>>(idx, prob, TK, K, E, nch, base, row_of_slot,
-                                                            token_of_row, prob_perm);
+    perm_rank_kernel<<<nch, kRankWarps * 32, 0, c.stream>>>(idx, prob, TK, K, E, nch, counts, offsets,
+                                                            row_of_slot, token_of_row, prob_perm);
   }
   return cudaGetLastError();
 }

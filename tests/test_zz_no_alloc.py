@@ -58,8 +58,8 @@ def test_noalloc_dispatch_matches_workspace_dispatch_on_two_calls_in_a_row(calls
 
 
 def test_noalloc_dispatch_rejects_shapes_beyond_its_fixed_scratch():
-    # E * ceil(T*K / 2048) = 256 * 513 > 131072: refused before anything is enqueued
-    shp = abi.MoeShape.of(2048 * 513 // 8, 1, 8, 64, 256, 64, "bf16")
+    # E * ceil(T*K / 2048) = 256 * 1025 > 262144: refused before anything is enqueued
+    shp = abi.MoeShape.of(2048 * 1025 // 8, 1, 8, 64, 256, 64, "bf16")
     with pytest.raises(abi.MoeError) as ei:
         abi.moe_dispatch_noalloc(shp, 16, 16, 16, 16, 16, 16, None, 16)
     assert ei.value.status == -9
