@@ -172,7 +172,7 @@ size_t align_up(size_t v) { return (v + 255) & ~size_t(255); }
 // Workspace carve-up.  Calls are ordered on one stream, so the regions used by
 // different calls may overlap.
 size_t ws_perm(const Dims& d) { return align_up(perm_workspace_bytes(d.TK, d.E)); }
-// dH [TK, 2F], dA [TK, F], then the wgrad GEMMs' per-expert tensor maps
+// dH [TK, 2F], dA [TK, F], then the wgrad GEMMs' per-expert tail tensor maps
 size_t ws_ffn_bwd_maps_offset(const Dims& d) { return align_up((size_t)d.TK * 3 * d.F * d.bx); }
 size_t ws_ffn_bwd(const Dims& d) { return ws_ffn_bwd_maps_offset(d) + align_up(gemm_tc_group_scratch_bytes(d.E)); }
 // Router weight gradient: split-K over the T tokens into at most kRouterSplits

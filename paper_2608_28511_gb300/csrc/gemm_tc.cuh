@@ -14,8 +14,10 @@
 //
 // Grouping: Group::M tiles never mix experts in an output row range (rows
 // past an expert's end are computed and dropped); Group::K reduces each
-// expert over its own row range through per-expert tensor maps (built on the
-// device by build_group_maps), so the copy engine zero-fills past the end.
+// expert over its own row range: whole 64-row k-blocks through the full
+// tensor maps, the last rows through a per-expert tail map (a host-encoded
+// template of exactly that many rows whose base build_group_maps moves), so
+// the copy engine zero-fills past the expert's end.
 //
 // Every mbarrier wait is bounded (kWaitLimitNs); on expiry the CTA sets the
 // device status word, drains its own copies and MMAs, frees TMEM and exits.
