@@ -262,7 +262,8 @@ def main() -> None:
     ap.add_argument("--ref-tokens", type=int, default=0, help="fixed oracle tokens per step (0 = sized to time)")
     ap.add_argument("--cpu-budget", type=float, default=15.0, help="seconds of CPU work for cpu_baseline")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--e2e-steps", type=int, default=10)
+    ap.add_argument("--e2e-steps", type=int, default=30,
+                    help="timed end-to-end steps (their first upload and last download are not overlapped)")
     ap.add_argument("--no-graph", action="store_true",
                     help="launch every kernel from the host each step instead of replaying a captured CUDA graph")
     ap.add_argument("--payload", default="bf16", choices=["bf16", "fp8"],
@@ -385,7 +386,7 @@ def main() -> None:
         torch.cuda.synchronize()
         e2e_ms = max_over_ranks(e_s.elapsed_time(e_e) / args.e2e_steps, world, "cuda")
         e2e = {"value": job_throughput(world, T, e2e_ms), "unit": UNIT, "h2d_bytes_per_step": h2d,
-               "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms,
+               "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms, "steps": args.e2e_steps,
                "api": "MoeLayer.run_host: step i+1's H2D and step i's D2H on two copy streams, overlapping compute"}
 
     # ---- per-kernel roofline from the live events
