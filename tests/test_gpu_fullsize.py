@@ -144,3 +144,30 @@ def test_full_size_parity(cfg):
     six = (L.x_perm.numel() + L.y_perm.numel() + L.dy_perm.numel() + L.dx_perm.numel()) * L.x_perm.element_size() \
         + (L.prob_perm.numel() + L.dprob_perm.numel()) * 4
     assert six == O.eq1_bytes(w.S, w.GBS, K, w.D, w.b_x, 4)
+
+
+def test_full_size_graph_and_host_pipeline_match_eager_bitwise():
+    """At the base workload, the two launch forms bench.py times reproduce the
+    eager step bit for bit: the step replayed as one CUDA graph, and
+    MoeLayer.run_host (host batches, copies overlapped with compute, one graph
+    per buffer set)."""
+    w = synth.get("C2")
+    L, inp = make_layer(w)
+    names = ("topk_idx", "row_of_slot", "x_perm", "h", "y", "dx_perm", "dw1", "dw2", "dx", "dw_router")
+    eager = {n: getattr(L, n).clone() for n in names}
+    g = L.capture()
+    for n in names:
+        getattr(L, n).zero_()
+    g.replay()
+    torch.cuda.synchronize()
+    for n in names:
+        assert torch.equal(getattr(L, n), eager[n]), n
+    x_h = inp["x"].pin_memory()
+    dy_h = inp["dy"].pin_memory()
+    y_h = torch.empty_like(x_h).pin_memory()
+    dx_h = torch.empty_like(x_h).pin_memory()
+    L.prepare_host_pipeline(graphs=True)
+    L.run_host([(x_h, dy_h, y_h, dx_h)] * 3)
+    torch.cuda.synchronize()
+    assert torch.equal(y_h, eager["y"].cpu())
+    assert torch.equal(dx_h, eager["dx"].cpu())
