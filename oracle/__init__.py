@@ -10,3 +10,4 @@ from .eq1 import *  # noqa: F401,F403
 from .router_sigmoid import *  # noqa: F401,F403
 from .shared import *  # noqa: F401,F403
 from .fp8 import *  # noqa: F401,F403
+from .nvfp4 import *  # noqa: F401,F403

@@ -206,3 +206,41 @@ def test_fp8_payload_mistakes_are_caught(monkeypatch):
     monkeypatch.setattr(F, "fp8_row_scale", scale_one_too_big)
     monkeypatch.setattr(oracle, "fp8_row_scale", scale_one_too_big)
     _expect_failure(PF.test_row_scale_is_the_smallest_fitting_power_of_two)
+
+
+def test_nvfp4_payload_mistakes_are_caught(monkeypatch):
+    import oracle.nvfp4 as N
+    import tests.test_oracle_nvfp4 as PN
+
+    # rounding ties away from zero instead of to the even code
+    def ties_away(v):
+        neg = v < 0
+        a = abs(v)
+        if a >= N.E2M1_MAX:
+            return N._CODES[-1] | (0x8 if neg else 0)
+        best = min(zip(N._CODES, N._VALS), key=lambda cv: (abs(cv[1] - a), -cv[1]))
+        return best[0] | (0x8 if neg else 0)
+    monkeypatch.setattr(N, "e2m1_quantize", ties_away)
+    monkeypatch.setattr(oracle, "e2m1_quantize", ties_away)
+    _expect_failure(PN.test_ties_to_even_saturation_and_sign)
+    monkeypatch.undo()
+
+    # the two codes of a byte swapped (element 2j in the high nibble)
+    real = N.nvfp4_quantize_rows
+
+    def swapped_nibbles(x):
+        codes, bsc, rsc = real(x)
+        return ((codes >> 4) | ((codes & 0xF) << 4)).astype(np.uint8), bsc, rsc
+    monkeypatch.setattr(N, "nvfp4_quantize_rows", swapped_nibbles)
+    monkeypatch.setattr(oracle, "nvfp4_quantize_rows", swapped_nibbles)
+    _expect_failure(PN.test_hand_computed_block)
+    monkeypatch.undo()
+
+    # block scale from the row maximum instead of the block's own maximum
+    def row_amax_scales(x):
+        codes, bsc, rsc = real(x)
+        bsc[:] = bsc.max(axis=1, keepdims=True)
+        return codes, bsc, rsc
+    monkeypatch.setattr(N, "nvfp4_quantize_rows", row_amax_scales)
+    monkeypatch.setattr(oracle, "nvfp4_quantize_rows", row_amax_scales)
+    _expect_failure(PN.test_round_trip_and_bf16_exactness)
