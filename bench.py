@@ -76,6 +76,8 @@ def kernel_work(name: str, w: synth.Workload, T: int, Fs: int = 0) -> tuple[str,
         "relusq_bwd": 3.0 * T * Fs * bx,
         "dispatch_fp8": T * D * bx + TK * D + 8 * TK,
         "dequant_rows": TK * D + TK * D * bx + 4 * TK,
+        "dispatch_nvfp4": T * D * bx + TK * (D // 2 + D // 16) + 8 * TK,
+        "dequant_nvfp4": TK * (D // 2 + D // 16) + TK * D * bx + 4 * TK,
         "pack_w1": 0.0,
     }
     return "hbm", float(byts.get(base, 0.0))
@@ -266,8 +268,9 @@ def main() -> None:
                     help="timed end-to-end steps (their first upload and last download are not overlapped)")
     ap.add_argument("--no-graph", action="store_true",
                     help="launch every kernel from the host each step instead of replaying a captured CUDA graph")
-    ap.add_argument("--payload", default="bf16", choices=["bf16", "fp8"],
-                    help="dispatch payload: bf16 rows, or FP8 E4M3 codes with a power-of-two scale per row")
+    ap.add_argument("--payload", default="bf16", choices=["bf16", "fp8", "nvfp4"],
+                    help="dispatch payload: bf16 rows, FP8 E4M3 codes with a power-of-two scale per row, or "
+                         "NVFP4 (E2M1 codes, an E4M3 scale per 16 elements, a power-of-two scale per row)")
     ap.add_argument("--shared-width", type=int, default=0,
                     help="hidden units of the ungated shared expert (0 = none; Sec. 5.2)")
     ap.add_argument("--router", default="softmax", choices=["softmax", "sigmoid"],

@@ -132,6 +132,30 @@ int moe_dispatch_fp8(const moe_shape_t* shape, const void* x, const int32_t* top
 int moe_dequant_rows(const moe_shape_t* shape, const void* x_perm_q, const float* x_scale_perm, void* x_perm,
                      void* stream);
 
+/* Dispatch with an NVFP4 payload (Sec. 1: lower-precision communication, b_x
+ * of Eq. 1; Sec. 6 names FP8 and NVFP4; readings NV1-NV3): the permutation and
+ * prob_perm as moe_dispatch, and each token's row x of x [T, D] (bf16 only;
+ * MOE_ERR_UNSUPPORTED otherwise) sent to its K rows in three arrays:
+ *   x_rscale_perm [TK] fp32: g = the smallest power of two 2^e, e >= -126,
+ *     with max_i |x_i| <= 6 * 448 * g (1 for an all-zero row);
+ *   x_bscale_perm [TK, D/16] E4M3 codes: per block b of 16 consecutive
+ *     elements, s_b = the E4M3 value nearest to the fp32 quotient
+ *     max_{i in b} |x_i| / (6 g), ties to even, saturating;
+ *   x_perm_q [TK, D/2] bytes: E2M1 codes (magnitudes 0, 0.5, 1, 1.5, 2, 3, 4,
+ *     6 and a sign bit), code_i = the E2M1 value nearest to the fp32 quotient
+ *     x_i / (s_b g), ties to even, saturating at +-6, zero where s_b = 0;
+ *     element 2j in the low nibble of byte j.
+ * The payload per routed slot is D/2 + D/16 + 4 + 4 bytes instead of 2 D + 4. */
+int moe_dispatch_nvfp4(const moe_shape_t* shape, const void* x, const int32_t* topk_idx, const float* topk_prob,
+                       int32_t* expert_offsets, int32_t* row_of_slot, int32_t* token_of_row, void* x_perm_q,
+                       uint8_t* x_bscale_perm, float* x_rscale_perm, float* prob_perm, void* ws, size_t ws_bytes,
+                       void* stream);
+
+/* The receiving side of moe_dispatch_nvfp4: x_perm[r, i] = value(code) * s_b * g
+ * in bf16 ([TK, D]; exact: at most 6 significant bits times a power of two). */
+int moe_dequant_nvfp4(const moe_shape_t* shape, const void* x_perm_q, const uint8_t* x_bscale_perm,
+                      const float* x_rscale_perm, void* x_perm, void* stream);
+
 /* Dispatch that allocates nothing and takes no workspace.  The paper has no
  * counterpart: this entry point exists for callers that cannot allocate
  * device memory when they call the layer -- a host framework that has already

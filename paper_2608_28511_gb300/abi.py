@@ -34,7 +34,7 @@ EXPORTS = (
     "moe_prof_reset", "moe_prof_count", "moe_prof_get", "moe_launch_count", "moe_dispatch_noalloc",
     "moe_ce_composition", "moe_ce_layer_pattern", "moe_route_sigmoid", "moe_route_sigmoid_bwd",
     "moe_shared_expert", "moe_shared_expert_bwd", "moe_expert_ffn_gather", "moe_expert_ffn_bwd_gather",
-    "moe_dispatch_fp8", "moe_dequant_rows",
+    "moe_dispatch_fp8", "moe_dequant_rows", "moe_dispatch_nvfp4", "moe_dequant_nvfp4",
 )
 
 
@@ -91,6 +91,8 @@ _SIGS = {
     "moe_expert_ffn_gather": ([_SHP] + [_VP] * 9 + [_SZ, _VP], ctypes.c_int),
     "moe_dispatch_fp8": ([_SHP] + [_VP] * 10 + [_SZ, _VP], ctypes.c_int),
     "moe_dequant_rows": ([_SHP, _VP, _VP, _VP, _VP], ctypes.c_int),
+    "moe_dispatch_nvfp4": ([_SHP] + [_VP] * 11 + [_SZ, _VP], ctypes.c_int),
+    "moe_dequant_nvfp4": ([_SHP, _VP, _VP, _VP, _VP, _VP], ctypes.c_int),
     "moe_expert_ffn_bwd_gather": ([_SHP] + [_VP] * 12 + [_SZ, _VP], ctypes.c_int),
     "moe_shared_expert": ([_SHP, _I32, _VP, _VP, _VP, _VP, _VP, _VP, _VP], ctypes.c_int),
     "moe_shared_expert_bwd": ([_SHP, _I32] + [_VP] * 11, ctypes.c_int),
@@ -206,6 +208,18 @@ def moe_dispatch_fp8(shape, x, topk_idx, topk_prob, expert_offsets, row_of_slot,
 def moe_dequant_rows(shape, x_perm_q, x_scale_perm, x_perm, stream=None):
     _check("moe_dequant_rows", lib().moe_dequant_rows(_shape(shape), _p(x_perm_q), _p(x_scale_perm), _p(x_perm),
                                                       _stream(stream)))
+
+
+def moe_dispatch_nvfp4(shape, x, topk_idx, topk_prob, expert_offsets, row_of_slot, token_of_row, x_perm_q,
+                       x_bscale_perm, x_rscale_perm, prob_perm, ws, stream=None):
+    _check("moe_dispatch_nvfp4", lib().moe_dispatch_nvfp4(
+        _shape(shape), _p(x), _p(topk_idx), _p(topk_prob), _p(expert_offsets), _p(row_of_slot), _p(token_of_row),
+        _p(x_perm_q), _p(x_bscale_perm), _p(x_rscale_perm), _p(prob_perm), _p(ws), _nbytes(ws), _stream(stream)))
+
+
+def moe_dequant_nvfp4(shape, x_perm_q, x_bscale_perm, x_rscale_perm, x_perm, stream=None):
+    _check("moe_dequant_nvfp4", lib().moe_dequant_nvfp4(_shape(shape), _p(x_perm_q), _p(x_bscale_perm),
+                                                        _p(x_rscale_perm), _p(x_perm), _stream(stream)))
 
 
 def moe_dispatch_noalloc(shape, x, topk_idx, topk_prob, expert_offsets, row_of_slot, token_of_row, x_perm,

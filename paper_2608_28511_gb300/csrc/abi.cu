@@ -417,6 +417,48 @@ int moe_dequant_rows(const moe_shape_t* shape, const void* x_perm_q, const float
   return MOE_OK;
 }
 
+int moe_dispatch_nvfp4(const moe_shape_t* shape, const void* x, const int32_t* topk_idx, const float* topk_prob,
+                       int32_t* expert_offsets, int32_t* row_of_slot, int32_t* token_of_row, void* x_perm_q,
+                       uint8_t* x_bscale_perm, float* x_rscale_perm, float* prob_perm, void* ws, size_t ws_bytes,
+                       void* stream) {
+  Dims d;
+  TRY(check_shape(shape, &d));
+  if (d.dt != DType::BF16) return MOE_ERR_UNSUPPORTED;
+  REQUIRE_PTR(x);
+  REQUIRE_PTR(topk_idx);
+  REQUIRE_PTR(topk_prob);
+  REQUIRE_PTR(expert_offsets);
+  REQUIRE_PTR(row_of_slot);
+  REQUIRE_PTR(token_of_row);
+  REQUIRE_PTR(x_perm_q);
+  REQUIRE_PTR(x_bscale_perm);
+  REQUIRE_PTR(x_rscale_perm);
+  REQUIRE_PTR(prob_perm);
+  REQUIRE_PTR(ws);
+  if (ws_bytes < ws_perm(d)) return MOE_ERR_WORKSPACE;
+  Ctx c;
+  TRY(get_ctx(stream, &c));
+  TRY_CUDA(launch_permutation(c, topk_idx, topk_prob, d.T, d.K, d.E, expert_offsets, row_of_slot, token_of_row,
+                              prob_perm, ws));
+  TRY_CUDA(launch_dispatch_nvfp4(c, x, row_of_slot, d.T, d.K, d.D, x_perm_q, x_bscale_perm, x_rscale_perm));
+  return MOE_OK;
+}
+
+int moe_dequant_nvfp4(const moe_shape_t* shape, const void* x_perm_q, const uint8_t* x_bscale_perm,
+                      const float* x_rscale_perm, void* x_perm, void* stream) {
+  Dims d;
+  TRY(check_shape(shape, &d));
+  if (d.dt != DType::BF16) return MOE_ERR_UNSUPPORTED;
+  REQUIRE_PTR(x_perm_q);
+  REQUIRE_PTR(x_bscale_perm);
+  REQUIRE_PTR(x_rscale_perm);
+  REQUIRE_PTR(x_perm);
+  Ctx c;
+  TRY(get_ctx(stream, &c));
+  TRY_CUDA(launch_dequant_nvfp4(c, x_perm_q, x_bscale_perm, x_rscale_perm, d.TK, d.D, x_perm));
+  return MOE_OK;
+}
+
 // The expert FFN with GEMM-1's A rows either read in order (x_rows = x_perm,
 // gather = NULL) or gathered from the dispatch input (x_rows = x [T, D],
 // gather = token_of_row).

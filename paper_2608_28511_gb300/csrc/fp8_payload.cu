@@ -87,18 +87,19 @@ __global__ void __launch_bounds__(256) dispatch_fp8_kernel(const uint4* __restri
   }
 }
 
-// x_perm[r] = codes[r] * scale[r] in bf16 (exact), 16 codes per thread step.
-__global__ void __launch_bounds__(256) dequant_rows_kernel(const uint4* __restrict__ xq,
-                                                           const float* __restrict__ scale, int64_t rows,
-                                                           int vpr16, uint4* __restrict__ out) {
-  const int64_t total = rows * vpr16;
+// x_perm[r] = codes[r] * scale[r] in bf16 (exact), 8 codes (one 16-byte
+// store) per thread step, so a warp writes 512 contiguous bytes.
+__global__ void __launch_bounds__(256) dequant_rows_kernel(const uint2* __restrict__ xq,
+                                                           const float* __restrict__ scale, int64_t rows, int vpr,
+                                                           uint4* __restrict__ out) {
+  const int64_t total = rows * vpr;
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total; i += (int64_t)gridDim.x * blockDim.x) {
-    const float s = __ldg(scale + i / vpr16);
-    const uint4 q = ld_stream(xq + i);
-    const uint32_t w[4] = {q.x, q.y, q.z, q.w};
-    float f[16];
+    const float s = __ldg(scale + i / vpr);
+    const uint2 q = __ldg(xq + i);
+    const uint32_t w[2] = {q.x, q.y};
+    float f[8];
 #pragma unroll
-    for (int h = 0; h < 4; ++h) {
+    for (int h = 0; h < 2; ++h) {
 #pragma unroll
       for (int j = 0; j < 2; ++j) {
         const __half2_raw hr = __nv_cvt_fp8x2_to_halfraw2((__nv_fp8x2_storage_t)(w[h] >> (16 * j)), __NV_E4M3);
@@ -107,8 +108,7 @@ __global__ void __launch_bounds__(256) dequant_rows_kernel(const uint4* __restri
         f[4 * h + 2 * j + 1] = v.y * s;
       }
     }
-    st_stream(out + 2 * i, pack16<bf16>(f));
-    st_stream(out + 2 * i + 1, pack16<bf16>(f + 8));
+    st_stream(out + i, pack16<bf16>(f));
   }
 }
 
@@ -138,11 +138,11 @@ cudaError_t launch_dispatch_fp8(const Ctx& c, const void* x, const int32_t* row_
 
 cudaError_t launch_dequant_rows(const Ctx& c, const void* xq, const float* scale, int64_t rows, int D, void* out) {
   if (rows == 0) return cudaSuccess;
-  const int vpr16 = D / 16;
-  const int64_t want = (rows * vpr16 + 255) / 256;
+  const int vpr = D / 8;
+  const int64_t want = (rows * vpr + 255) / 256;
   const int blocks = (int)(want < (int64_t)c.num_sms * 16 ? want : (int64_t)c.num_sms * 16);
   KernelScope ks("dequant_rows", c.stream);
-  dequant_rows_kernel<<<blocks, 256, 0, c.stream>>>((const uint4*)xq, scale, rows, vpr16, (uint4*)out);
+  dequant_rows_kernel<<<blocks, 256, 0, c.stream>>>((const uint2*)xq, scale, rows, vpr, (uint4*)out);
   return cudaGetLastError();
 }
 

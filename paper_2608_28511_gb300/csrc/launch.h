@@ -97,6 +97,14 @@ cudaError_t launch_dispatch_fp8(const Ctx& c, const void* x, const int32_t* row_
                                 void* xq, float* scale_perm);
 cudaError_t launch_dequant_rows(const Ctx& c, const void* xq, const float* scale, int64_t rows, int D, void* out);
 
+// nvfp4_payload.cu: E2M1 codes [TK, D/2] (two per byte), E4M3 block scales
+// [TK, D/16] and power-of-two row scales [TK] of the bf16 rows x [T, D]
+// written to each token's K rows; and their bf16 values.
+cudaError_t launch_dispatch_nvfp4(const Ctx& c, const void* x, const int32_t* row_of_slot, int64_t T, int K, int D,
+                                  void* xq, uint8_t* bscale, float* rscale);
+cudaError_t launch_dequant_nvfp4(const Ctx& c, const void* xq, const uint8_t* bscale, const float* rscale,
+                                 int64_t rows, int D, void* out);
+
 // swiglu.cu: dH [rows, 2F] (packed) from dA [rows, F] and the saved h [rows, 2F].
 cudaError_t launch_swiglu_bwd(const Ctx& c, DType dt, const void* dA, const void* h, int64_t rows, int F,
                               void* dH);

@@ -34,7 +34,9 @@ class MoeLayer:
     128-row tile).
     ``payload="fp8"`` dispatches the hidden rows as FP8 E4M3 codes with one
     power-of-two scale per row (b_x = 1) and dequantizes them on arrival;
-    the gradient passes the quantization unchanged.
+    the gradient passes the quantization unchanged.  ``payload="nvfp4"``
+    sends E2M1 codes with one E4M3 scale per 16 elements and one power-of-two
+    scale per row (b_x = 1/2 plus the scales) the same way.
     """
 
     def __init__(self, S, GBS, K, D, E, F, dtype="bf16", H=0, device="cuda", router="softmax", aux_coef=1e-4,
@@ -43,7 +45,7 @@ class MoeLayer:
             raise ValueError(f"unknown router {router!r}")
         self.router = router
         self.gather = bool(gather)
-        if payload not in ("bf16", "fp8") or (payload == "fp8" and (gather or dtype != "bf16")):
+        if payload not in ("bf16", "fp8", "nvfp4") or (payload != "bf16" and (gather or dtype != "bf16")):
             raise ValueError(f"payload {payload!r} with gather={gather}, dtype={dtype}")
         self.payload = payload
         self.aux_coef = float(aux_coef)
@@ -84,6 +86,9 @@ class MoeLayer:
         self.x_perm = None if self.gather else e(TK, D)
         self.x_perm_q = e(TK, D, d=torch.uint8) if payload == "fp8" else None
         self.x_scale_perm = e(TK, d=f32) if payload == "fp8" else None
+        self.x_perm_q4 = e(TK, D // 2, d=torch.uint8) if payload == "nvfp4" else None
+        self.x_bscale_perm = e(TK, D // 16, d=torch.uint8) if payload == "nvfp4" else None
+        self.x_rscale_perm = e(TK, d=f32) if payload == "nvfp4" else None
         self.prob_perm = e(TK, d=f32)
         self.h = e(TK, 2 * F)
         self.act = e(TK, F)
@@ -152,6 +157,11 @@ class MoeLayer:
             abi.moe_dispatch_fp8(s, xd, self.topk_idx, self.topk_prob, self.expert_offsets, self.row_of_slot,
                                  self.token_of_row, self.x_perm_q, self.x_scale_perm, self.prob_perm, self.ws, stream)
             abi.moe_dequant_rows(s, self.x_perm_q, self.x_scale_perm, self.x_perm, stream)
+        elif self.payload == "nvfp4":
+            abi.moe_dispatch_nvfp4(s, xd, self.topk_idx, self.topk_prob, self.expert_offsets, self.row_of_slot,
+                                   self.token_of_row, self.x_perm_q4, self.x_bscale_perm, self.x_rscale_perm,
+                                   self.prob_perm, self.ws, stream)
+            abi.moe_dequant_nvfp4(s, self.x_perm_q4, self.x_bscale_perm, self.x_rscale_perm, self.x_perm, stream)
         else:
             abi.moe_dispatch(s, xd, self.topk_idx, self.topk_prob, self.expert_offsets, self.row_of_slot,
                              self.token_of_row, self.x_perm, self.prob_perm, self.ws, stream)
