@@ -11,6 +11,7 @@ replicas).  Prints one JSON line on rank 0.
 from __future__ import annotations
 
 import argparse
+import dataclasses
 import json
 import os
 import statistics
@@ -229,6 +230,25 @@ def run_reference(args, w: synth.Workload) -> None:
 # Multi-rank host logic (weak scaling: every rank its own tokens)
 # ---------------------------------------------------------------------------
 
+def step_statistics(per_step):
+    """Per-step spread of the timed pass: the median, and the filtered mean of
+    the paper's training-cost estimator (Empirical results, "Evaluation
+    axes"): steps slower than the current mean + 1.5 standard deviations are
+    removed, repeatedly, until none is.  The headline stays the plain mean
+    over all K steps."""
+    kept = list(per_step)
+    while len(kept) > 1:
+        mean = sum(kept) / len(kept)
+        sd = (sum((t - mean) ** 2 for t in kept) / len(kept)) ** 0.5
+        nxt = [t for t in kept if t <= mean + 1.5 * sd]
+        if len(nxt) == len(kept):
+            break
+        kept = nxt
+    return {"median_ms": round(statistics.median(per_step), 4),
+            "filtered_mean_ms": round(sum(kept) / len(kept), 4), "dropped": len(per_step) - len(kept),
+            "min_ms": round(min(per_step), 4), "max_ms": round(max(per_step), 4)}
+
+
 def rank_seed(w: synth.Workload, rank: int) -> int:
     """Seed of rank ``rank``'s token batch: ranks hold disjoint synthetic batches."""
     return w.seed + rank
@@ -260,6 +280,8 @@ def main() -> None:
     ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--workload", default="C2")
+    ap.add_argument("--seed", type=int, default=None,
+                    help="input seed of rank 0 (default: the workload's own, 0); seeds 1 and 2 give the variance check")
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--ref-tokens", type=int, default=0, help="fixed oracle tokens per step (0 = sized to time)")
     ap.add_argument("--cpu-budget", type=float, default=15.0, help="seconds of CPU work for cpu_baseline")
@@ -278,6 +300,8 @@ def main() -> None:
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
     w = synth.get(args.workload)
+    if args.seed is not None:
+        w = dataclasses.replace(w, seed=args.seed)
 
     if args.impl == "reference":
         run_reference(args, w)
@@ -354,15 +378,18 @@ def main() -> None:
         launches = (abi.moe_launch_count() - n0) // args.steps
         abi.moe_prof_enable(False)
         prof = abi.moe_prof_read() if kernel_events else {}
-        step_ms = sum(s.elapsed_time(e) for s, e in zip(ev_s, ev_e)) / args.steps
-        return step_ms, wall, launches, prof
+        per_step = [s.elapsed_time(e) for s, e in zip(ev_s, ev_e)]
+        return per_step, wall, launches, prof
 
     clocks = ClockSampler(local)
-    step_ms, wall, _, _ = timed_steps(kernel_events=False)
+    per_step, wall, _, _ = timed_steps(kernel_events=False)
     clk = clocks.stop()
+    step_ms = sum(per_step) / len(per_step)
+    step_stats = step_statistics(per_step)
     t_max = max_over_ranks(step_ms, world, "cuda")
     assert abi.moe_check_device_status() == 0
-    step_ms_ev, _, launches, prof = timed_steps(kernel_events=True)
+    per_step_ev, _, launches, prof = timed_steps(kernel_events=True)
+    step_ms_ev = sum(per_step_ev) / len(per_step_ev)
     assert abi.moe_check_device_status() == 0
 
     # ---- end to end through the public API with host buffers
@@ -461,6 +488,7 @@ def main() -> None:
             "clocks": clk,
             "wall_s_timed_region": wall,
             "ms_per_step_kernel_events_pass": round(step_ms_ev, 4),
+            "step_stats": step_stats,
             "kernels": detail,
         }
         print(json.dumps(line), flush=True)

@@ -68,3 +68,15 @@ def test_reference_arm_runs_only_on_rank_zero(monkeypatch, capsys):
 
 def test_job_throughput_is_weak_scaling():
     assert bench.job_throughput(4, 8192, 2.0) == pytest.approx(4 * bench.job_throughput(1, 8192, 2.0))
+
+
+def test_step_statistics_filters_outliers_iteratively():
+    """The filtered mean removes steps above mean + 1.5 sd until none is left:
+    one slow step (10) is removed first; the next pass then removes the
+    moderate one (2) that the first pass's wide sd let through."""
+    steps = [1.0] * 20 + [2.0, 10.0]
+    st = bench.step_statistics(steps)
+    assert st["dropped"] == 2
+    assert st["filtered_mean_ms"] == 1.0
+    assert st["median_ms"] == 1.0 and st["max_ms"] == 10.0
+    assert bench.step_statistics([1.0, 1.0, 1.0])["dropped"] == 0
