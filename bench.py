@@ -69,6 +69,7 @@ def kernel_work(name: str, w: synth.Workload, T: int, Fs: int = 0) -> tuple[str,
         "combine": (TK + T) * D * bx + 8 * TK,
         "combine_bwd": (T + 2 * TK) * D * bx + 12 * TK,
         "dispatch_bwd": (TK + T) * D * bx + 8 * TK,
+        "dispatch_route_bwd": (TK + T) * D * bx + E * D * bx + 8 * TK + 8 * T * K + 4 * T * E + 2 * T * E,
         "route_dz": T * K * 12 + T * E * 6,
         "select_sigmoid": T * E * 4 + T * K * 8,
         "balance_finalize": 0.0,
@@ -453,7 +454,7 @@ def main() -> None:
                 "frac": achieved / peak, "traffic": traffic, "peak_note": f"HBM copy, of {peaks['source']}"}
 
     exp_ms = sum(v["ms_per_step"] for k, v in kernels.items() if k.startswith("ffn") or k == "swiglu_bwd")
-    perm_names = ("dispatch_rows", "combine", "combine_bwd", "dispatch_bwd")
+    perm_names = ("dispatch_rows", "combine", "combine_bwd", "dispatch_bwd", "dispatch_route_bwd")
     perm_ms = sum(v["ms_per_step"] for k, v in kernels.items() if k in perm_names)
     detail = {k: {"ms_per_step": round(v["ms_per_step"], 4),
                   ("TFLOP/s" if v["bound"] == "tensor" else "GB/s"):

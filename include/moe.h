@@ -245,6 +245,22 @@ int moe_route_bwd(const moe_shape_t* shape, const void* x, const void* w_router,
                   const float* topk_prob, const float* dtopk_prob, void* dx, float* dw_router, float* dlogits,
                   void* ws, size_t ws_bytes, void* stream);
 
+/* moe_dispatch_bwd followed by moe_route_bwd in one pass over the tokens, for
+ * a layer without latent projection (H = 0; MOE_ERR_UNSUPPORTED otherwise),
+ * where the router reads the dispatch input x [T, D].  dlogits is nonzero only
+ * on each token's K chosen experts, so dlogits . w_router for token t is a sum
+ * of K rows of w_router [E, D]; it is added while the K rows of dx_perm are
+ * summed:
+ *   dx[t] = sum_k dx_perm[r_k] + sum_k dlogits[t, e_k] w_router[e_k]
+ * with fp32 accumulation and ONE rounding (the two separate calls round dx
+ * twice), dtopk_prob and dlogits as the two calls (dlogits bit-identical),
+ * dw_router = dlogits^T . x as moe_route_bwd.  dx [T, D] is overwritten.
+ * Workspace as moe_route_bwd. */
+int moe_dispatch_route_bwd(const moe_shape_t* shape, const void* dx_perm, const float* dprob_perm,
+                           const int32_t* row_of_slot, const void* x, const void* w_router, const int32_t* topk_idx,
+                           const float* topk_prob, void* dx, float* dtopk_prob, float* dlogits, float* dw_router,
+                           void* ws, size_t ws_bytes, void* stream);
+
 /* Sigmoid router with expert bias and the sequence-level balance loss
  * (Sec. 5.2 experimental details; the paper gives no formulas, readings S1-S3):
  *   logits[T, E] = x[T, Din] . w_router^T (fp32, no logit bias);

@@ -34,7 +34,7 @@ EXPORTS = (
     "moe_prof_reset", "moe_prof_count", "moe_prof_get", "moe_launch_count", "moe_dispatch_noalloc",
     "moe_ce_composition", "moe_ce_layer_pattern", "moe_route_sigmoid", "moe_route_sigmoid_bwd",
     "moe_shared_expert", "moe_shared_expert_bwd", "moe_expert_ffn_gather", "moe_expert_ffn_bwd_gather",
-    "moe_dispatch_fp8", "moe_dequant_rows", "moe_dispatch_nvfp4", "moe_dequant_nvfp4",
+    "moe_dispatch_fp8", "moe_dequant_rows", "moe_dispatch_nvfp4", "moe_dequant_nvfp4", "moe_dispatch_route_bwd",
 )
 
 
@@ -85,6 +85,7 @@ _SIGS = {
     "moe_expert_ffn_bwd": ([_SHP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _SZ, _VP], ctypes.c_int),
     "moe_dispatch_bwd": ([_SHP, _VP, _VP, _VP, _VP, _VP, _VP], ctypes.c_int),
     "moe_route_bwd": ([_SHP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _SZ, _VP], ctypes.c_int),
+    "moe_dispatch_route_bwd": ([_SHP] + [_VP] * 12 + [_SZ, _VP], ctypes.c_int),
     "moe_route_sigmoid": ([_SHP, _VP, _VP, _VP, _F32, _VP, _VP, _VP, _VP, _VP, _VP, _SZ, _VP], ctypes.c_int),
     "moe_route_sigmoid_bwd": ([_SHP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _F32, _F32, _VP, _VP, _VP, _VP, _SZ, _VP],
                               ctypes.c_int),
@@ -271,6 +272,13 @@ def moe_expert_ffn_bwd(shape, dy_perm, x_perm, h_save, act_save, expert_offsets,
 def moe_dispatch_bwd(shape, dx_perm, dprob_perm, row_of_slot, dx, dtopk_prob, stream=None):
     _check("moe_dispatch_bwd", lib().moe_dispatch_bwd(_shape(shape), _p(dx_perm), _p(dprob_perm), _p(row_of_slot),
                                                       _p(dx), _p(dtopk_prob), _stream(stream)))
+
+
+def moe_dispatch_route_bwd(shape, dx_perm, dprob_perm, row_of_slot, x, w_router, topk_idx, topk_prob, dx,
+                           dtopk_prob, dlogits, dw_router, ws, stream=None):
+    _check("moe_dispatch_route_bwd", lib().moe_dispatch_route_bwd(
+        _shape(shape), _p(dx_perm), _p(dprob_perm), _p(row_of_slot), _p(x), _p(w_router), _p(topk_idx),
+        _p(topk_prob), _p(dx), _p(dtopk_prob), _p(dlogits), _p(dw_router), _p(ws), _nbytes(ws), _stream(stream)))
 
 
 def moe_route_bwd(shape, x, w_router, topk_idx, topk_prob, dtopk_prob, dx, dw_router, dlogits, ws, stream=None):

@@ -760,7 +760,7 @@ int moe_dispatch_bwd(const moe_shape_t* shape, const void* dx_perm, const float*
 // dx[T, Din] += dz . w_router and dw_router = dz^T . x, from dz [T, E] fp32 and
 // (bf16 inputs) its bf16 copy at the start of the workspace.
 static int router_grad_gemms(const Ctx& c, const Dims& d, const void* x, const void* w_router, const float* dlogits,
-                      void* dx, float* dw_router, void* ws) {
+                      void* dx, float* dw_router, void* ws, bool dgrad = true) {
   void* dz16 = d.dt == DType::BF16 ? ws : nullptr;
   // dx += dz . w_router   (M = T, N = Din, K = E)
   GemmDesc a;
@@ -808,7 +808,7 @@ static int router_grad_gemms(const Ctx& c, const Dims& d, const void* x, const v
     if (gemm_tc_supports(a16)) a = a16;
     if (gemm_tc_supports(b16)) b = b16;
   }
-  if (d.T > 0) TRY_CUDA(gemm(c, a, "router_dgrad_tc", "router_dgrad_simt"));
+  if (dgrad && d.T > 0) TRY_CUDA(gemm(c, a, "router_dgrad_tc", "router_dgrad_simt"));
   const int splits = d.dt == DType::BF16 ? router_splits(d, c.num_sms) : 1;
   if (splits > 1) {
     // split-K: partial products of equal token ranges, then their in-order sum
@@ -854,6 +854,34 @@ int moe_route_bwd(const moe_shape_t* shape, const void* x, const void* w_router,
   void* dz16 = d.dt == DType::BF16 ? ws : nullptr;
   TRY_CUDA(launch_route_dz(c, topk_idx, topk_prob, dtopk_prob, d.T, d.E, d.K, dlogits, dz16));
   return router_grad_gemms(c, d, x, w_router, dlogits, dx, dw_router, ws);
+}
+
+int moe_dispatch_route_bwd(const moe_shape_t* shape, const void* dx_perm, const float* dprob_perm,
+                           const int32_t* row_of_slot, const void* x, const void* w_router, const int32_t* topk_idx,
+                           const float* topk_prob, void* dx, float* dtopk_prob, float* dlogits, float* dw_router,
+                           void* ws, size_t ws_bytes, void* stream) {
+  Dims d;
+  TRY(check_shape(shape, &d));
+  if (d.H) return MOE_ERR_UNSUPPORTED;  // the router reads x [T, H], the dispatch x_lat [T, D]
+  REQUIRE_PTR(dx_perm);
+  REQUIRE_PTR(dprob_perm);
+  REQUIRE_PTR(row_of_slot);
+  REQUIRE_PTR(x);
+  REQUIRE_PTR(w_router);
+  REQUIRE_PTR(topk_idx);
+  REQUIRE_PTR(topk_prob);
+  REQUIRE_PTR(dx);
+  REQUIRE_PTR(dtopk_prob);
+  REQUIRE_PTR(dlogits);
+  REQUIRE_PTR(dw_router);
+  REQUIRE_PTR(ws);
+  if (ws_bytes < ws_route_bwd(d)) return MOE_ERR_WORKSPACE;
+  Ctx c;
+  TRY(get_ctx(stream, &c));
+  void* dz16 = d.dt == DType::BF16 ? ws : nullptr;
+  TRY_CUDA(launch_dispatch_route_bwd(c, d.dt, dx_perm, dprob_perm, row_of_slot, topk_idx, topk_prob, w_router, d.T,
+                                     d.K, d.E, d.D, dx, dtopk_prob, dlogits, dz16));
+  return router_grad_gemms(c, d, x, w_router, dlogits, dx, dw_router, ws, /*dgrad=*/false);
 }
 
 int moe_route_sigmoid(const moe_shape_t* shape, const void* x, const void* w_router, const float* expert_bias,

@@ -88,6 +88,12 @@ cudaError_t launch_combine_bwd(const Ctx& c, DType dt, const void* dy, const voi
                                float* dprob_perm);
 cudaError_t launch_dispatch_bwd(const Ctx& c, DType dt, const void* dx_perm, const float* dprob_perm,
                                 const int32_t* row_of_slot, int64_t T, int K, int D, void* dx, float* dprob);
+// permute.cu: the dispatch backward fused with the softmax router's dz and
+// dx += dz . w_router (w_router [E, D]); dz16 (bf16 copy of dz) may be NULL.
+cudaError_t launch_dispatch_route_bwd(const Ctx& c, DType dt, const void* dx_perm, const float* dprob_perm,
+                                      const int32_t* row_of_slot, const int32_t* idx, const float* prob,
+                                      const void* w_router, int64_t T, int K, int E, int D, void* dx, float* dprob,
+                                      float* dz, void* dz16);
 cudaError_t launch_pack_w1(const Ctx& c, DType dt, const void* w_gate, const void* w_up, int E, int F, int D,
                            void* w1);
 

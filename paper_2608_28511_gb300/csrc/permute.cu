@@ -376,6 +376,119 @@ cudaError_t launch_dispatch_bwd(const Ctx& c, DType dt, const void* dx_perm, con
   return cudaGetLastError();
 }
 
+// Dispatch backward fused with the softmax router's backward, for a router
+// that reads the dispatch input itself (no latent projection).  dz is nonzero
+// only on a token's K selected experts, so dz . W_r for token t is a sum of
+// K rows of W_r [E, D], the same shape as the sum over its K dX_perm rows.
+// Per token t (one warp):
+//   dprob[t, k] = dprob_perm[row_k];
+//   dz[t, e_k]  = p_k (dprob[t, k] - sum_j p_j dprob[t, j]), 0 elsewhere
+//                 (the same reduction tree as route_dz_kernel, so the same bits);
+//   dx[t]       = sum_k dX_perm[row_k] + sum_k dz[t, e_k] W_r[e_k]
+//                 (fp32 accumulation, rounded once).
+// dz16 (bf16 copy of dz, for the router weight gradient) may be NULL.
+template <typename T, int KM>
+__global__ void __launch_bounds__(256, KM <= 8 ? 3 : 1) dispatch_route_bwd_kernel(
+    const uint4* __restrict__ dx_perm, const float* __restrict__ dprob_perm, const int32_t* __restrict__ row_of_slot,
+    const int32_t* __restrict__ idx, const float* __restrict__ prob, const uint4* __restrict__ w_router, int64_t Tn,
+    int K, int E, int vpr, uint4* __restrict__ dx, float* __restrict__ dprob, float* __restrict__ dz,
+    bf16* __restrict__ dz16, uint32_t* err) {
+  constexpr int NV = Vec<T>::N;
+  const int lane = threadIdx.x & 31;
+  const int64_t t = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  if (t >= Tn) return;
+  int32_t rows[KM];
+  load_rows<KM>(row_of_slot, t, K, rows);
+  int my_e = -1;
+  float my_p = 0.f, my_dp = 0.f;
+  if (lane < K) {
+    my_e = __ldg(idx + t * K + lane);
+    my_p = __ldg(prob + t * K + lane);
+    my_dp = __ldg(dprob_perm + __ldg(row_of_slot + t * K + lane));
+  }
+  float cdot = my_p * my_dp;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) cdot += __shfl_xor_sync(0xffffffffu, cdot, off);
+  const float my_dz = my_p * (my_dp - cdot);
+  int ek[KM];
+  float dzk[KM];
+#pragma unroll
+  for (int k = 0; k < KM; ++k) {
+    ek[k] = __shfl_sync(0xffffffffu, my_e, k);
+    dzk[k] = __shfl_sync(0xffffffffu, my_dz, k);
+    if (k < K && (ek[k] < 0 || ek[k] >= E)) {  // an expert index outside [0, E): recorded, its row skipped
+      if (lane == 0) set_error(err, kErrIndex);
+      ek[k] = -1;
+    }
+  }
+  for (int v = lane; v < vpr; v += 32) {
+    // the K dX_perm rows (HBM) first, then the K rows of W_r (L2-resident):
+    // one set of K vectors in registers at a time keeps three blocks per SM
+    uint4 raw[KM];
+#pragma unroll
+    for (int k = 0; k < KM; ++k)
+      if (k < K) raw[k] = ld_stream(dx_perm + (int64_t)rows[k] * vpr + v);
+    float acc[NV];
+#pragma unroll
+    for (int i = 0; i < NV; ++i) acc[i] = 0.f;
+#pragma unroll
+    for (int k = 0; k < KM; ++k) {
+      if (k < K) {
+        float f[NV];
+        unpack16<T>(raw[k], f);
+#pragma unroll
+        for (int i = 0; i < NV; ++i) acc[i] += f[i];
+      }
+    }
+#pragma unroll
+    for (int k = 0; k < KM; ++k)
+      if (k < K && ek[k] >= 0) raw[k] = ld_keep(w_router + (int64_t)ek[k] * vpr + v);
+#pragma unroll
+    for (int k = 0; k < KM; ++k) {
+      if (k < K && ek[k] >= 0) {
+        float f[NV];
+        unpack16<T>(raw[k], f);
+#pragma unroll
+        for (int i = 0; i < NV; ++i) acc[i] = fmaf(dzk[k], f[i], acc[i]);
+      }
+    }
+    st_stream(dx + t * vpr + v, pack16<T>(acc));
+  }
+  if (lane < K) dprob[t * K + lane] = my_dp;
+  for (int e0 = 0; e0 < E; e0 += 32) {
+    const int e = e0 + lane;
+    float val = 0.f;
+#pragma unroll
+    for (int k = 0; k < KM; ++k)
+      if (k < K && ek[k] == e) val = dzk[k];
+    if (e < E) {
+      dz[t * E + e] = val;
+      if (dz16) dz16[t * E + e] = __float2bfloat16_rn(val);
+    }
+  }
+}
+
+cudaError_t launch_dispatch_route_bwd(const Ctx& c, DType dt, const void* dx_perm, const float* dprob_perm,
+                                      const int32_t* row_of_slot, const int32_t* idx, const float* prob,
+                                      const void* w_router, int64_t T, int K, int E, int D, void* dx, float* dprob,
+                                      float* dz, void* dz16) {
+  if (T == 0) return cudaSuccess;
+  const int warps = 8;
+  const int vpr = (int)((int64_t)D * dsize(dt) / 16);
+  const unsigned grid = (unsigned)((T + warps - 1) / warps);
+  KernelScope ks("dispatch_route_bwd", c.stream);
+  if (dt == DType::BF16) {
+    MOE_DISPATCH_KM(K, (dispatch_route_bwd_kernel<bf16, KM><<<grid, 32 * warps, 0, c.stream>>>(
+                           (const uint4*)dx_perm, dprob_perm, row_of_slot, idx, prob, (const uint4*)w_router, T, K,
+                           E, vpr, (uint4*)dx, dprob, dz, (bf16*)dz16, c.err)));
+  } else {
+    MOE_DISPATCH_KM(K, (dispatch_route_bwd_kernel<float, KM><<<grid, 32 * warps, 0, c.stream>>>(
+                           (const uint4*)dx_perm, dprob_perm, row_of_slot, idx, prob, (const uint4*)w_router, T, K,
+                           E, vpr, (uint4*)dx, dprob, dz, (bf16*)dz16, c.err)));
+  }
+  return cudaGetLastError();
+}
+
 // w1[e, 128 i + c] = w_gate[e, 64 i + c] for c < 64, w_up[e, 64 i + c - 64] otherwise.
 __global__ void __launch_bounds__(256) pack_w1_kernel(const uint4* __restrict__ wg, const uint4* __restrict__ wu,
                                                       int64_t rows_total, int F, int vpr, uint4* __restrict__ w1) {

@@ -202,13 +202,18 @@ class MoeLayer:
             abi.moe_dispatch_bwd(s, self.dx_perm, self.dprob_perm, self.row_of_slot, self.dx_lat, self.dprob, stream)
             abi.moe_latent_proj_bwd(s, self.H, self.D, self.dx_lat, self.x, self.w_down, self.dx, False,
                                     self.dw_down, self.ws, stream)
+        elif self.router == "softmax":
+            # one pass: dispatch backward, dlogits and dx += dlogits . w_router
+            abi.moe_dispatch_route_bwd(s, self.dx_perm, self.dprob_perm, self.row_of_slot, self.x, self.w_router,
+                                       self.topk_idx, self.topk_prob, self.dx, self.dprob, self.dlogits,
+                                       self.dw_router, self.ws, stream)
         else:
             abi.moe_dispatch_bwd(s, self.dx_perm, self.dprob_perm, self.row_of_slot, self.dx, self.dprob, stream)
         if self.router == "sigmoid":
             abi.moe_route_sigmoid_bwd(s, self.x, self.w_router, self.logits, self.topk_idx, self.topk_prob,
                                       self.dprob, self.aux_f, self.aux_coef, self.aux_grad, self.dx, self.dw_router,
                                       self.dlogits, self.ws, stream)
-        else:
+        elif self.H:
             abi.moe_route_bwd(s, self.x, self.w_router, self.topk_idx, self.topk_prob, self.dprob, self.dx,
                               self.dw_router, self.dlogits, self.ws, stream)
         if self.shared_F:

@@ -39,6 +39,26 @@ def test_every_declared_symbol_is_exported(L):
     assert sorted(L.EXPORTS) == syms
 
 
+def _prototypes():
+    """{name: number of parameters} of every function include/moe.h declares."""
+    text = open(os.path.join(ROOT, "include", "moe.h")).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    out = {}
+    for m in re.finditer(r"\b(moe_[a-z0-9_]+)\s*\(([^)]*)\)\s*;", text):
+        params = m.group(2).strip()
+        out[m.group(1)] = 0 if params in ("", "void") else params.count(",") + 1
+    return out
+
+
+def test_binding_signatures_match_the_header(L):
+    """Each ctypes signature of the binding has as many arguments as the C
+    prototype (a missing or extra argument would shift every later one)."""
+    protos = _prototypes()
+    assert sorted(protos) == sorted(L.EXPORTS)
+    for name, (args, _res) in L._SIGS.items():
+        assert len(args) == protos[name], (name, len(args), protos[name])
+
+
 def test_version_and_strerror(L):
     assert L.moe_version() >= 100
     for st in (0, -1, -2, -3, -4, -5, -6, -7, -8):
