@@ -1,9 +1,11 @@
 """Full-size parity of the next-step rows at the base workload (T=8192, D=2048,
 E=64, K=6, F=1024), in the launch configuration bench.py times for them:
-the sigmoid router (``--router sigmoid``) and the shared expert
-(``--shared-width 2688``).  Index work on every token, statistics and router
-gradients over all tokens, the shared expert on sampled tokens and its whole
-weight gradients; tolerances as in the other parity tests."""
+the sigmoid router (``--router sigmoid``), the shared expert
+(``--shared-width 2688``) and the FP8 and NVFP4 payloads (``--payload``).
+Index work and payload codes on every token, statistics and router gradients
+over all tokens, the shared expert and the layer output on sampled tokens, the
+shared expert's whole weight gradients; tolerances as in the other parity
+tests."""
 import numpy as np
 import pytest
 import torch
@@ -103,6 +105,41 @@ def test_fp8_payload_full_size():
     rng = np.random.default_rng(11)
     toks = np.unique(np.concatenate([[0, W.T - 1], rng.choice(W.T, 48, replace=False)]))
     x_deq = O.fp8_dequantize_rows(codes[toks], scales[toks])
+    idx = i64(L.topk_idx)[toks]
+    prob = f64(L.topk_prob)[toks]
+    wg, wu, w2 = (_w64(inp[k]) for k in ("w_gate", "w_up", "w2"))
+    y_ref = np.zeros((len(toks), W.D))
+    for i in range(len(toks)):
+        for k in range(W.K):
+            e = idx[i, k]
+            g, u = x_deq[i] @ wg[e].T, x_deq[i] @ wu[e].T
+            y_ref[i] += prob[i, k] * ((O.silu(g) * u) @ w2[e].T)
+    assert rel_frob(f64(L.y)[toks], y_ref) <= REL_FROB
+
+
+def test_nvfp4_payload_full_size():
+    """The NVFP4 dispatch payload at the base workload (``--payload nvfp4``):
+    every token's E2M1 codes, E4M3 block scales and row scale at all K of its
+    rows, bit for bit against the oracle's quantization of the GPU's own
+    dispatch input; the dequantized rows exactly; sampled tokens' layer output
+    within the layer tolerance, from the dequantized rows (readings NV1-NV3)."""
+    from paper_2608_28511_gb300.layer import MoeLayer
+    inp = synth.make_inputs(W)
+    L = MoeLayer(W.S, W.GBS, W.K, W.D, W.E, W.F, W.dtype, W.H, payload="nvfp4")
+    L.load(inp)
+    L.forward()
+    L.backward()
+    torch.cuda.synchronize()
+    x = _w64(inp["x"])
+    codes, bsc, rsc = O.nvfp4_quantize_rows(x)
+    tor = i64(L.token_of_row)
+    assert np.array_equal(L.x_perm_q4.cpu().numpy(), codes[tor])
+    assert np.array_equal(L.x_bscale_perm.cpu().numpy(), bsc[tor])
+    assert np.array_equal(f64(L.x_rscale_perm), rsc[tor])
+    assert np.array_equal(f64(L.x_perm), O.nvfp4_dequantize_rows(codes, bsc, rsc)[tor])
+    rng = np.random.default_rng(12)
+    toks = np.unique(np.concatenate([[0, W.T - 1], rng.choice(W.T, 48, replace=False)]))
+    x_deq = O.nvfp4_dequantize_rows(codes[toks], bsc[toks], rsc[toks])
     idx = i64(L.topk_idx)[toks]
     prob = f64(L.topk_prob)[toks]
     wg, wu, w2 = (_w64(inp[k]) for k in ("w_gate", "w_up", "w2"))
