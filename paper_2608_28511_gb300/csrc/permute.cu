@@ -27,9 +27,18 @@ __global__ void __launch_bounds__(256) perm_hist_kernel(const int32_t* __restric
   __syncthreads();
   const int64_t s0 = (int64_t)blockIdx.x * kChunk;
   const int64_t s1 = min(TK, s0 + kChunk);
-  for (int64_t s = s0 + threadIdx.x; s < s1; s += blockDim.x) {
-    const int e = idx[s];
-    if (e >= 0 && e < E) atomicAdd(&h[e], 1);
+  // every load of the thread's kChunk / 256 slots in flight before the counts
+  constexpr int kPer = kChunk / 256;
+  int ev[kPer];
+#pragma unroll
+  for (int i = 0; i < kPer; ++i) {
+    const int64_t s = s0 + i * 256 + threadIdx.x;
+    ev[i] = s < s1 ? __ldg(idx + s) : 0;
+  }
+#pragma unroll
+  for (int i = 0; i < kPer; ++i) {
+    if (s0 + i * 256 + threadIdx.x >= s1) continue;
+    if (ev[i] >= 0 && ev[i] < E) atomicAdd(&h[ev[i]], 1);
     else set_error(err, kErrIndex);
   }
   __syncthreads();
@@ -57,6 +66,7 @@ __global__ void __launch_bounds__(kRankWarps * 32) perm_rank_kernel(
   for (int e = threadIdx.x; e < E; e += blockDim.x) {
     const int32_t* row = counts + (int64_t)e * nchunks;
     int before = 0, all = 0;
+#pragma unroll 8
     for (int c = 0; c < nchunks; ++c) {
       const int v = row[c];
       before += c < (int)blockIdx.x ? v : 0;
@@ -81,10 +91,19 @@ __global__ void __launch_bounds__(kRankWarps * 32) perm_rank_kernel(
   const int64_t c0 = (int64_t)blockIdx.x * kChunk;
   const int64_t w0 = c0 + (int64_t)warp * kSub;
   const int64_t w1 = min(TK, w0 + kSub);
-  for (int64_t s = w0 + lane; s < w1; s += 32) {
-    const int e = idx[s];
-    if (e >= 0 && e < E) atomicAdd(&cnt[warp * E + e], 1);
+  // the warp's kSub expert indices and probabilities, all loads in flight at
+  // once (expert -1 past the end)
+  int ev[kSub / 32];
+  float pv[kSub / 32];
+#pragma unroll
+  for (int i = 0; i < kSub / 32; ++i) {
+    const int64_t s = w0 + i * 32 + lane;
+    ev[i] = s < w1 ? __ldg(idx + s) : -1;
+    pv[i] = s < w1 ? __ldg(prob + s) : 0.f;
   }
+#pragma unroll
+  for (int i = 0; i < kSub / 32; ++i)
+    if (ev[i] >= 0 && ev[i] < E) atomicAdd(&cnt[warp * E + ev[i]], 1);
   __syncthreads();
   for (int e = threadIdx.x; e < E; e += blockDim.x) {
     int run = tot[e] + pre[e];
@@ -96,10 +115,10 @@ __global__ void __launch_bounds__(kRankWarps * 32) perm_rank_kernel(
   }
   __syncthreads();
   const unsigned lt = (1u << lane) - 1u;
-  for (int64_t b = w0; b < w0 + kSub; b += 32) {
-    const int64_t s = b + lane;
-    int e = -1;
-    if (s < w1) e = idx[s];
+#pragma unroll
+  for (int i = 0; i < kSub / 32; ++i) {
+    const int64_t s = w0 + i * 32 + lane;
+    const int e = ev[i];
     const bool valid = (s < w1) && e >= 0 && e < E;
     const unsigned peers = __match_any_sync(0xffffffffu, valid ? e : -1);
     const int rank = __popc(peers & lt);
@@ -109,7 +128,7 @@ __global__ void __launch_bounds__(kRankWarps * 32) perm_rank_kernel(
       const int row = here + rank;
       row_of_slot[s] = row;
       token_of_row[row] = (int32_t)(s / K);
-      prob_perm[row] = prob[s];
+      prob_perm[row] = pv[i];
       if (rank == __popc(peers) - 1) cnt[warp * E + e] = here + __popc(peers);
     } else if (s < w1) {
       row_of_slot[s] = 0;  // keeps downstream gathers in bounds; the status word is set
