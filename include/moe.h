@@ -261,6 +261,27 @@ int moe_dispatch_route_bwd(const moe_shape_t* shape, const void* dx_perm, const 
                            const float* topk_prob, void* dx, float* dtopk_prob, float* dlogits, float* dw_router,
                            void* ws, size_t ws_bytes, void* stream);
 
+/* The backward tail of a LatentMoE layer with the softmax router (H > 0,
+ * bf16, (D + E) a multiple of 8; MOE_ERR_UNSUPPORTED otherwise), in place of
+ * moe_dispatch_bwd into dx_lat, moe_latent_proj_bwd of the down-projection
+ * and moe_route_bwd.  The router reads x [T, H], so its dx term is not a sum
+ * of rows of the dispatch gradient.  Instead both gradients into x come out
+ * of ONE product over the concatenated reduction dimension:
+ *   dx_cat = [dx_lat | dz] [T, D + E] (bf16, written: the dispatch backward's
+ *   sums in columns 0 .. D-1, the bf16 copy of dlogits in D .. D+E-1) times
+ *   w_down_router [D + E, H] = w_down [D, H] stacked on w_router [E, H]
+ *   (one contiguous array: the caller keeps the two weights there),
+ *   dx = dx_lat . w_down + dlogits . w_router  (fp32 accumulation, one rounding;
+ *   the separate calls round twice).
+ * dtopk_prob, dlogits, dw_down = dx_lat^T . x and dw_router = dlogits^T . x
+ * (fp32) are as the separate calls compute them.  dx [T, H] is overwritten.
+ * Workspace: moe_workspace_size(). */
+int moe_latent_route_bwd(const moe_shape_t* shape, const void* dx_perm, const float* dprob_perm,
+                         const int32_t* row_of_slot, const void* x, const void* w_down_router,
+                         const int32_t* topk_idx, const float* topk_prob, void* dx_cat, void* dx,
+                         float* dtopk_prob, float* dlogits, float* dw_down, float* dw_router, void* ws,
+                         size_t ws_bytes, void* stream);
+
 /* Sigmoid router with expert bias and the sequence-level balance loss
  * (Sec. 5.2 experimental details; the paper gives no formulas, readings S1-S3):
  *   logits[T, E] = x[T, Din] . w_router^T (fp32, no logit bias);

@@ -35,6 +35,7 @@ EXPORTS = (
     "moe_ce_composition", "moe_ce_layer_pattern", "moe_route_sigmoid", "moe_route_sigmoid_bwd",
     "moe_shared_expert", "moe_shared_expert_bwd", "moe_expert_ffn_gather", "moe_expert_ffn_bwd_gather",
     "moe_dispatch_fp8", "moe_dequant_rows", "moe_dispatch_nvfp4", "moe_dequant_nvfp4", "moe_dispatch_route_bwd",
+    "moe_latent_route_bwd",
 )
 
 
@@ -86,6 +87,7 @@ _SIGS = {
     "moe_dispatch_bwd": ([_SHP, _VP, _VP, _VP, _VP, _VP, _VP], ctypes.c_int),
     "moe_route_bwd": ([_SHP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _SZ, _VP], ctypes.c_int),
     "moe_dispatch_route_bwd": ([_SHP] + [_VP] * 12 + [_SZ, _VP], ctypes.c_int),
+    "moe_latent_route_bwd": ([_SHP] + [_VP] * 14 + [_SZ, _VP], ctypes.c_int),
     "moe_route_sigmoid": ([_SHP, _VP, _VP, _VP, _F32, _VP, _VP, _VP, _VP, _VP, _VP, _SZ, _VP], ctypes.c_int),
     "moe_route_sigmoid_bwd": ([_SHP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _F32, _F32, _VP, _VP, _VP, _VP, _SZ, _VP],
                               ctypes.c_int),
@@ -279,6 +281,14 @@ def moe_dispatch_route_bwd(shape, dx_perm, dprob_perm, row_of_slot, x, w_router,
     _check("moe_dispatch_route_bwd", lib().moe_dispatch_route_bwd(
         _shape(shape), _p(dx_perm), _p(dprob_perm), _p(row_of_slot), _p(x), _p(w_router), _p(topk_idx),
         _p(topk_prob), _p(dx), _p(dtopk_prob), _p(dlogits), _p(dw_router), _p(ws), _nbytes(ws), _stream(stream)))
+
+
+def moe_latent_route_bwd(shape, dx_perm, dprob_perm, row_of_slot, x, w_down_router, topk_idx, topk_prob, dx_cat,
+                         dx, dtopk_prob, dlogits, dw_down, dw_router, ws, stream=None):
+    _check("moe_latent_route_bwd", lib().moe_latent_route_bwd(
+        _shape(shape), _p(dx_perm), _p(dprob_perm), _p(row_of_slot), _p(x), _p(w_down_router), _p(topk_idx),
+        _p(topk_prob), _p(dx_cat), _p(dx), _p(dtopk_prob), _p(dlogits), _p(dw_down), _p(dw_router), _p(ws),
+        _nbytes(ws), _stream(stream)))
 
 
 def moe_route_bwd(shape, x, w_router, topk_idx, topk_prob, dtopk_prob, dx, dw_router, dlogits, ws, stream=None):

@@ -757,11 +757,35 @@ int moe_dispatch_bwd(const moe_shape_t* shape, const void* dx_perm, const float*
   return MOE_OK;
 }
 
+static GemmDesc dense_desc(Epi epi, int64_t M, int64_t N, int64_t K, const void* A, DType at, int64_t sa_m,
+                           int64_t sa_k, const void* B, DType bt, int64_t sb_n, int64_t sb_k, void* C, DType ct,
+                           int64_t ldc) {
+  GemmDesc g;
+  g.group = Group::Dense;
+  g.epi = epi;
+  g.M = M;
+  g.N = N;
+  g.K = K;
+  g.A = A;
+  g.a_type = at;
+  g.sa_m = sa_m;
+  g.sa_k = sa_k;
+  g.B = B;
+  g.b_type = bt;
+  g.sb_n = sb_n;
+  g.sb_k = sb_k;
+  g.C = C;
+  g.c_type = ct;
+  g.ldc = ldc;
+  return g;
+}
+
 // dx[T, Din] += dz . w_router and dw_router = dz^T . x, from dz [T, E] fp32 and
-// (bf16 inputs) its bf16 copy at the start of the workspace.
+// (bf16 inputs) its bf16 copy dz16 (rows dz16_ld elements apart); scratch
+// holds the weight gradient's split-K partials and tail maps.
 static int router_grad_gemms(const Ctx& c, const Dims& d, const void* x, const void* w_router, const float* dlogits,
-                      void* dx, float* dw_router, void* ws, bool dgrad = true) {
-  void* dz16 = d.dt == DType::BF16 ? ws : nullptr;
+                             void* dx, float* dw_router, const void* dz16, int64_t dz16_ld, void* scratch,
+                             bool dgrad = true) {
   // dx += dz . w_router   (M = T, N = Din, K = E)
   GemmDesc a;
   a.group = Group::Dense;
@@ -803,8 +827,10 @@ static int router_grad_gemms(const Ctx& c, const Dims& d, const void* x, const v
     GemmDesc a16 = a, b16 = b;
     a16.A = dz16;
     a16.a_type = DType::BF16;
+    a16.sa_m = dz16_ld;
     b16.A = dz16;
     b16.a_type = DType::BF16;
+    b16.sa_k = dz16_ld;
     if (gemm_tc_supports(a16)) a = a16;
     if (gemm_tc_supports(b16)) b = b16;
   }
@@ -820,9 +846,9 @@ static int router_grad_gemms(const Ctx& c, const Dims& d, const void* x, const v
     bs.max_rows = d.T;
     bs.A = dz16;
     bs.a_type = DType::BF16;
-    bs.C = static_cast<char*>(ws) + ws_route_dz(d);
+    bs.C = scratch;
     bs.sc_g = (int64_t)d.E * d.Din;
-    bs.scratch = static_cast<char*>(ws) + ws_route_dz(d) + ws_route_parts(d);
+    bs.scratch = static_cast<char*>(scratch) + ws_route_parts(d);
     if (gemm_tc_supports(bs)) {
       TRY_CUDA(launch_gemm_tc(c, bs, "router_wgrad_tc"));
       TRY_CUDA(launch_sum_splits(c, static_cast<const float*>(bs.C), splits, (int64_t)d.E * d.Din, dw_router));
@@ -853,7 +879,8 @@ int moe_route_bwd(const moe_shape_t* shape, const void* x, const void* w_router,
   TRY(get_ctx(stream, &c));
   void* dz16 = d.dt == DType::BF16 ? ws : nullptr;
   TRY_CUDA(launch_route_dz(c, topk_idx, topk_prob, dtopk_prob, d.T, d.E, d.K, dlogits, dz16));
-  return router_grad_gemms(c, d, x, w_router, dlogits, dx, dw_router, ws);
+  return router_grad_gemms(c, d, x, w_router, dlogits, dx, dw_router, ws, d.E,
+                           static_cast<char*>(ws) + ws_route_dz(d));
 }
 
 int moe_dispatch_route_bwd(const moe_shape_t* shape, const void* dx_perm, const float* dprob_perm,
@@ -881,7 +908,51 @@ int moe_dispatch_route_bwd(const moe_shape_t* shape, const void* dx_perm, const 
   void* dz16 = d.dt == DType::BF16 ? ws : nullptr;
   TRY_CUDA(launch_dispatch_route_bwd(c, d.dt, dx_perm, dprob_perm, row_of_slot, topk_idx, topk_prob, w_router, d.T,
                                      d.K, d.E, d.D, dx, dtopk_prob, dlogits, dz16));
-  return router_grad_gemms(c, d, x, w_router, dlogits, dx, dw_router, ws, /*dgrad=*/false);
+  return router_grad_gemms(c, d, x, w_router, dlogits, dx, dw_router, ws, d.E,
+                           static_cast<char*>(ws) + ws_route_dz(d), /*dgrad=*/false);
+}
+
+int moe_latent_route_bwd(const moe_shape_t* shape, const void* dx_perm, const float* dprob_perm,
+                         const int32_t* row_of_slot, const void* x, const void* w_down_router,
+                         const int32_t* topk_idx, const float* topk_prob, void* dx_cat, void* dx,
+                         float* dtopk_prob, float* dlogits, float* dw_down, float* dw_router, void* ws,
+                         size_t ws_bytes, void* stream) {
+  Dims d;
+  TRY(check_shape(shape, &d));
+  if (!d.H || d.dt != DType::BF16 || (d.D + d.E) % 8) return MOE_ERR_UNSUPPORTED;
+  REQUIRE_PTR(dx_perm);
+  REQUIRE_PTR(dprob_perm);
+  REQUIRE_PTR(row_of_slot);
+  REQUIRE_PTR(x);
+  REQUIRE_PTR(w_down_router);
+  REQUIRE_PTR(topk_idx);
+  REQUIRE_PTR(topk_prob);
+  REQUIRE_PTR(dx_cat);
+  REQUIRE_PTR(dx);
+  REQUIRE_PTR(dtopk_prob);
+  REQUIRE_PTR(dlogits);
+  REQUIRE_PTR(dw_down);
+  REQUIRE_PTR(dw_router);
+  REQUIRE_PTR(ws);
+  if (ws_bytes < ws_route_bwd(d)) return MOE_ERR_WORKSPACE;
+  Ctx c;
+  TRY(get_ctx(stream, &c));
+  const int64_t ldk = d.D + d.E;                   // row length of [dx_lat | dz16]
+  bf16* cat = static_cast<bf16*>(dx_cat);
+  void* scratch = ws;
+  const bf16* w_router = static_cast<const bf16*>(w_down_router) + (int64_t)d.D * d.H;
+  TRY_CUDA(launch_dispatch_bwd(c, d.dt, dx_perm, dprob_perm, row_of_slot, d.T, d.K, d.D, cat, dtopk_prob, ldk));
+  TRY_CUDA(launch_route_dz(c, topk_idx, topk_prob, dtopk_prob, d.T, d.E, d.K, dlogits, cat + d.D, ldk));
+  if (d.T > 0) {
+    // dx = dx_lat . w_down + dz . w_router   (M = T, N = H, K = D + E, one rounding)
+    GemmDesc a = dense_desc(Epi::Store, d.T, d.H, ldk, cat, d.dt, ldk, 1, w_down_router, d.dt, 1, d.H, dx, d.dt,
+                            d.H);
+    TRY_CUDA(gemm(c, a, "latent_dgrad_tc", "latent_dgrad_simt"));
+  }
+  // dw_down = dx_lat^T . x   (M = D, N = H, K = T)
+  GemmDesc b = dense_desc(Epi::Store, d.D, d.H, d.T, cat, d.dt, 1, ldk, x, d.dt, 1, d.H, dw_down, DType::F32, d.H);
+  TRY_CUDA(gemm(c, b, "latent_wgrad_tc", "latent_wgrad_simt"));
+  return router_grad_gemms(c, d, x, w_router, dlogits, dx, dw_router, cat + d.D, ldk, scratch, /*dgrad=*/false);
 }
 
 int moe_route_sigmoid(const moe_shape_t* shape, const void* x, const void* w_router, const float* expert_bias,
@@ -949,7 +1020,8 @@ int moe_route_sigmoid_bwd(const moe_shape_t* shape, const void* x, const void* w
   void* dz16 = d.dt == DType::BF16 ? ws : nullptr;
   TRY_CUDA(launch_route_dz_sigmoid(c, logits, topk_idx, topk_prob, dtopk_prob, aux_f, d.T, d.S, d.GBS, d.E, d.K,
                                    aux_coef, aux_grad, dlogits, dz16));
-  return router_grad_gemms(c, d, x, w_router, dlogits, dx, dw_router, ws);
+  return router_grad_gemms(c, d, x, w_router, dlogits, dx, dw_router, ws, d.E,
+                           static_cast<char*>(ws) + ws_route_dz(d));
 }
 
 int moe_latent_proj(const moe_shape_t* shape, int32_t n_in, int32_t n_out, const void* in, const void* w,
@@ -1044,28 +1116,6 @@ int moe_latent_proj_bwd(const moe_shape_t* shape, int32_t n_in, int32_t n_out, c
 }
 
 // A dense C(m, n) = sum_k A(m, k) B(n, k) descriptor (element strides).
-static GemmDesc dense_desc(Epi epi, int64_t M, int64_t N, int64_t K, const void* A, DType at, int64_t sa_m,
-                           int64_t sa_k, const void* B, DType bt, int64_t sb_n, int64_t sb_k, void* C, DType ct,
-                           int64_t ldc) {
-  GemmDesc g;
-  g.group = Group::Dense;
-  g.epi = epi;
-  g.M = M;
-  g.N = N;
-  g.K = K;
-  g.A = A;
-  g.a_type = at;
-  g.sa_m = sa_m;
-  g.sa_k = sa_k;
-  g.B = B;
-  g.b_type = bt;
-  g.sb_n = sb_n;
-  g.sb_k = sb_k;
-  g.C = C;
-  g.c_type = ct;
-  g.ldc = ldc;
-  return g;
-}
 
 int moe_shared_expert(const moe_shape_t* shape, int32_t F_s, const void* x, const void* w_s1, const void* w_s2,
                       void* h_save, void* act_save, void* y, void* stream) {

@@ -53,9 +53,10 @@ constexpr int kMaxE = 256;
 cudaError_t launch_topk(const Ctx& c, const float* logits, int64_t T, int E, int K, int32_t* idx, float* prob);
 // out[i] = sum over s of part[s * n + i], s = 0 .. S-1 in order (fp32).
 cudaError_t launch_sum_splits(const Ctx& c, const float* part, int S, int64_t n, float* out);
-// dz[T, E] fp32 (fully written) and optionally a bf16 copy.
+// dz[T, E] fp32 (fully written) and optionally a bf16 copy whose rows are
+// ld16 elements apart (0: E).
 cudaError_t launch_route_dz(const Ctx& c, const int32_t* idx, const float* prob, const float* dprob, int64_t T,
-                            int E, int K, float* dz, void* dz_bf16);
+                            int E, int K, float* dz, void* dz_bf16, int64_t ld16 = 0);
 
 // ---------------------------------------------------------------------------
 // router_sigmoid.cu
@@ -86,8 +87,10 @@ cudaError_t launch_combine(const Ctx& c, DType dt, const void* y_perm, const flo
 cudaError_t launch_combine_bwd(const Ctx& c, DType dt, const void* dy, const void* y_perm, const float* prob_perm,
                                const int32_t* row_of_slot, int64_t T, int K, int D, void* dy_perm,
                                float* dprob_perm);
+// dx rows ldx elements apart (0: D).
 cudaError_t launch_dispatch_bwd(const Ctx& c, DType dt, const void* dx_perm, const float* dprob_perm,
-                                const int32_t* row_of_slot, int64_t T, int K, int D, void* dx, float* dprob);
+                                const int32_t* row_of_slot, int64_t T, int K, int D, void* dx, float* dprob,
+                                int64_t ldx = 0);
 // permute.cu: the dispatch backward fused with the softmax router's dz and
 // dx += dz . w_router (w_router [E, D]); dz16 (bf16 copy of dz) may be NULL.
 cudaError_t launch_dispatch_route_bwd(const Ctx& c, DType dt, const void* dx_perm, const float* dprob_perm,

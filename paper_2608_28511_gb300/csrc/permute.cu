@@ -341,13 +341,13 @@ cudaError_t launch_combine_bwd(const Ctx& c, DType dt, const void* dy, const voi
   return cudaGetLastError();
 }
 
-// Dispatch backward: dx[t] = sum_k dX_perm[row_k] (fp32 accumulation);
-// dprob[t, k] = dprob_perm[row_k].
+// Dispatch backward: dx[t] = sum_k dX_perm[row_k] (fp32 accumulation; dx
+// rows ldv 16-byte vectors apart); dprob[t, k] = dprob_perm[row_k].
 template <typename T, int KM>
 __global__ void __launch_bounds__(256) dispatch_bwd_kernel(const uint4* __restrict__ dx_perm,
                                                            const float* __restrict__ dprob_perm,
                                                            const int32_t* __restrict__ row_of_slot, int64_t Tn,
-                                                           int K, int vpr, uint4* __restrict__ dx,
+                                                           int K, int vpr, int64_t ldv, uint4* __restrict__ dx,
                                                            float* __restrict__ dprob) {
   constexpr int NV = Vec<T>::N;
   const int lane = threadIdx.x & 31;
@@ -372,25 +372,27 @@ __global__ void __launch_bounds__(256) dispatch_bwd_kernel(const uint4* __restri
         for (int i = 0; i < NV; ++i) acc[i] += f[i];
       }
     }
-    st_stream(dx + t * vpr + v, pack16<T>(acc));
+    st_stream(dx + t * ldv + v, pack16<T>(acc));
   }
   // the probability gradients last, off the path of the row loads
   if (lane < K) dprob[t * K + lane] = __ldg(dprob_perm + row_of_slot[t * K + lane]);
 }
 
 cudaError_t launch_dispatch_bwd(const Ctx& c, DType dt, const void* dx_perm, const float* dprob_perm,
-                                const int32_t* row_of_slot, int64_t T, int K, int D, void* dx, float* dprob) {
+                                const int32_t* row_of_slot, int64_t T, int K, int D, void* dx, float* dprob,
+                                int64_t ldx) {
   if (T == 0) return cudaSuccess;
   const int warps = 8;
   const int vpr = (int)((int64_t)D * dsize(dt) / 16);
+  const int64_t ldv = (ldx > 0 ? ldx : D) * (int64_t)dsize(dt) / 16;
   const unsigned grid = (unsigned)((T + warps - 1) / warps);
   KernelScope ks("dispatch_bwd", c.stream);
   if (dt == DType::BF16) {
     MOE_DISPATCH_KM(K, (dispatch_bwd_kernel<bf16, KM><<<grid, 32 * warps, 0, c.stream>>>(
-                           (const uint4*)dx_perm, dprob_perm, row_of_slot, T, K, vpr, (uint4*)dx, dprob)));
+                           (const uint4*)dx_perm, dprob_perm, row_of_slot, T, K, vpr, ldv, (uint4*)dx, dprob)));
   } else {
     MOE_DISPATCH_KM(K, (dispatch_bwd_kernel<float, KM><<<grid, 32 * warps, 0, c.stream>>>(
-                           (const uint4*)dx_perm, dprob_perm, row_of_slot, T, K, vpr, (uint4*)dx, dprob)));
+                           (const uint4*)dx_perm, dprob_perm, row_of_slot, T, K, vpr, ldv, (uint4*)dx, dprob)));
   }
   return cudaGetLastError();
 }

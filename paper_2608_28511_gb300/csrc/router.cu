@@ -73,7 +73,8 @@ cudaError_t launch_topk(const Ctx& c, const float* logits, int64_t T, int E, int
 __global__ void __launch_bounds__(256) route_dz_kernel(const int32_t* __restrict__ idx,
                                                        const float* __restrict__ prob,
                                                        const float* __restrict__ dprob, int64_t T, int E, int K,
-                                                       float* __restrict__ dz, bf16* __restrict__ dz_bf16) {
+                                                       float* __restrict__ dz, bf16* __restrict__ dz_bf16,
+                                                       int64_t ld16) {
   const int lane = threadIdx.x & 31;
   const int64_t t = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   if (t >= T) return;
@@ -98,18 +99,19 @@ __global__ void __launch_bounds__(256) route_dz_kernel(const int32_t* __restrict
     }
     if (e < E) {
       dz[t * E + e] = val;
-      if (dz_bf16) dz_bf16[t * E + e] = __float2bfloat16_rn(val);
+      if (dz_bf16) dz_bf16[t * ld16 + e] = __float2bfloat16_rn(val);
     }
   }
 }
 
 cudaError_t launch_route_dz(const Ctx& c, const int32_t* idx, const float* prob, const float* dprob, int64_t T,
-                            int E, int K, float* dz, void* dz_bf16) {
+                            int E, int K, float* dz, void* dz_bf16, int64_t ld16) {
   if (T == 0) return cudaSuccess;
   const int warps = 8;
   dim3 grid((unsigned)((T + warps - 1) / warps)), block(32 * warps);
   KernelScope ks("route_dz", c.stream);
-  route_dz_kernel<<<grid, block, 0, c.stream>>>(idx, prob, dprob, T, E, K, dz, (bf16*)dz_bf16);
+  route_dz_kernel<<<grid, block, 0, c.stream>>>(idx, prob, dprob, T, E, K, dz, (bf16*)dz_bf16,
+                                                 ld16 > 0 ? ld16 : E);
   return cudaGetLastError();
 }
 

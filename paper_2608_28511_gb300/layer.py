@@ -61,8 +61,12 @@ class MoeLayer:
         f32, i32 = torch.float32, torch.int32
         e = lambda *s, d=dt: torch.empty(*s, dtype=d, device=dev)  # noqa: E731
         Din = self.Din
-        # weights
-        self.w_router = e(E, Din)
+        # weights; a LatentMoE layer with the softmax router keeps w_down [D, H]
+        # and w_router [E, H] in one [D + E, H] array, which its backward reads
+        # as one operand (moe_latent_route_bwd)
+        self.latent_fused = bool(H) and router == "softmax" and dtype == "bf16" and (D + E) % 8 == 0
+        self.w_down_router = e(D + E, H) if self.latent_fused else None
+        self.w_router = self.w_down_router[D:] if self.latent_fused else e(E, Din)
         self.w1 = e(E, 2 * F, D)
         self.w2 = e(E, D, F)
         self.bias = None
@@ -70,7 +74,7 @@ class MoeLayer:
         self.shared_F = Fs = int(shared_F)
         self.w_s1 = e(Fs, self.Din) if Fs else None
         self.w_s2 = e(self.Din, Fs) if Fs else None
-        self.w_down = e(D, H) if H else None
+        self.w_down = (self.w_down_router[:D] if self.latent_fused else e(D, H)) if H else None
         self.w_upp = e(H, D) if H else None
         # forward
         self.x = e(T, Din)
@@ -108,7 +112,9 @@ class MoeLayer:
         self.dx_perm = e(TK, D)
         self.dw1 = e(E, 2 * F, D, d=f32)
         self.dw2 = e(E, D, F, d=f32)
-        self.dx_lat = e(T, D) if H else None
+        # fused LatentMoE tail: [dx_lat | bf16 dlogits] in one [T, D + E] array
+        self.dx_cat = e(T, D + E) if self.latent_fused else None
+        self.dx_lat = (self.dx_cat[:, :D] if self.latent_fused else e(T, D)) if H else None
         self.dprob = e(T, K, d=f32)
         self.dx = e(T, Din)
         self.dlogits = e(T, E, d=f32)
@@ -198,7 +204,12 @@ class MoeLayer:
         else:
             abi.moe_expert_ffn_bwd(s, self.dy_perm, self.x_perm, self.h, self.act, self.expert_offsets, self.w1,
                                    self.w2, self.dx_perm, self.dw1, self.dw2, self.ws, stream)
-        if self.H:
+        if self.latent_fused:
+            # dispatch backward, dlogits, dw_down, dw_router and dx from one product over [dx_lat | dz]
+            abi.moe_latent_route_bwd(s, self.dx_perm, self.dprob_perm, self.row_of_slot, self.x, self.w_down_router,
+                                     self.topk_idx, self.topk_prob, self.dx_cat, self.dx, self.dprob, self.dlogits,
+                                     self.dw_down, self.dw_router, self.ws, stream)
+        elif self.H:
             abi.moe_dispatch_bwd(s, self.dx_perm, self.dprob_perm, self.row_of_slot, self.dx_lat, self.dprob, stream)
             abi.moe_latent_proj_bwd(s, self.H, self.D, self.dx_lat, self.x, self.w_down, self.dx, False,
                                     self.dw_down, self.ws, stream)
@@ -213,7 +224,7 @@ class MoeLayer:
             abi.moe_route_sigmoid_bwd(s, self.x, self.w_router, self.logits, self.topk_idx, self.topk_prob,
                                       self.dprob, self.aux_f, self.aux_coef, self.aux_grad, self.dx, self.dw_router,
                                       self.dlogits, self.ws, stream)
-        elif self.H:
+        elif self.H and not self.latent_fused:
             abi.moe_route_bwd(s, self.x, self.w_router, self.topk_idx, self.topk_prob, self.dprob, self.dx,
                               self.dw_router, self.dlogits, self.ws, stream)
         if self.shared_F:
