@@ -46,14 +46,18 @@ def _peaks() -> dict:
 # once and each result written once.
 # ---------------------------------------------------------------------------
 
-def kernel_work(name: str, w: synth.Workload, T: int, Fs: int = 0) -> tuple[str, float]:
+def kernel_work(name: str, w: synth.Workload, T: int, Fs: int = 0, latent_fused: bool = False) -> tuple[str, float]:
+    """(bound, algorithmic work per launch) of a library kernel: flops for the
+    tensor-core GEMMs, bytes for the rest.  latent_fused: the LatentMoE dgrad
+    also carries the router's dz W_r term (reduction over D + E)."""
     TK, D, E, K, F, bx = T * w.K, w.D, w.E, w.K, w.F, w.b_x
     Din = w.H if w.H else D
     base = name.rsplit("_", 1)[0] if name.endswith(("_tc", "_simt")) else name
     flops = {
         "ffn1_swiglu": 4.0 * TK * D * F, "ffn2": 2.0 * TK * F * D, "ffn2_dgrad": 2.0 * TK * D * F,
         "ffn2_wgrad": 2.0 * TK * D * F, "ffn1_dgrad": 4.0 * TK * F * D, "ffn1_wgrad": 4.0 * TK * F * D,
-        "latent_fwd": 2.0 * T * w.H * D, "latent_dgrad": 2.0 * T * w.H * D, "latent_wgrad": 2.0 * T * w.H * D,
+        "latent_fwd": 2.0 * T * w.H * D, "latent_dgrad": 2.0 * T * w.H * (D + (E if latent_fused else 0)),
+        "latent_wgrad": 2.0 * T * w.H * D,
         "router_dgrad": 2.0 * T * Din * E, "router_wgrad": 2.0 * T * Din * E,
         "shared_fc1": 2.0 * T * Din * Fs, "shared_fc2": 2.0 * T * Fs * Din,
         "shared_fc2_dgrad": 2.0 * T * Din * Fs, "shared_fc1_dgrad": 2.0 * T * Fs * Din,
@@ -424,7 +428,7 @@ def main() -> None:
     peaks = _peaks()
     kernels = {}
     for name, (n, ms) in prof.items():
-        bound, work = kernel_work(name, w, T, args.shared_width)
+        bound, work = kernel_work(name, w, T, args.shared_width, L.latent_fused)
         per_launch_ms = ms / max(n, 1)
         kernels[name] = {"launches_per_step": n / args.steps, "ms_per_step": ms / args.steps,
                          "bound": bound, "work_per_launch": work, "avg_launch_ms": per_launch_ms}

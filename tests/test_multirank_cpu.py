@@ -80,3 +80,23 @@ def test_step_statistics_filters_outliers_iteratively():
     assert st["filtered_mean_ms"] == 1.0
     assert st["median_ms"] == 1.0 and st["max_ms"] == 10.0
     assert bench.step_statistics([1.0, 1.0, 1.0])["dropped"] == 0
+
+
+def test_every_timed_kernel_has_algorithmic_work():
+    """Each kernel the library times (KernelScope names and the tensor-core
+    GEMM names in the C sources) has a roofline entry in bench.kernel_work,
+    except the few that do no algorithmic work of the method."""
+    import glob
+    import re
+    import synth
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    names = set()
+    for f in glob.glob(os.path.join(root, "paper_2608_28511_gb300", "csrc", "*.cu")):
+        text = open(f).read()
+        names |= set(re.findall(r'KernelScope ks\("([a-z0-9_]+)"', text))
+        names |= set(re.findall(r'"([a-z0-9_]+_tc)"', text))
+    no_work = {"group_maps", "sum_splits", "pack_w1", "perm_zero", "balance_finalize"}
+    w = synth.get("C4")
+    missing = [n for n in sorted(names - no_work) if bench.kernel_work(n, w, w.T, 2688)[1] <= 0]
+    assert not missing, missing
+    assert len(names) >= 30
