@@ -115,3 +115,27 @@ def test_python_binding_raises_on_error(L):
     with pytest.raises(L.MoeError) as ei:
         L.moe_workspace_size(shp)
     assert ei.value.status == -1
+
+
+def test_layer_buffer_layout_for_the_fused_backward_tails(L):
+    """Host-side layout of MoeLayer (CPU tensors, no launch): with H > 0 and
+    the softmax router, w_down and w_router are consecutive row ranges of one
+    [D + E, H] array and dx_lat is the first D columns of [dx_lat | dz]; the
+    other configurations keep separate arrays."""
+    import torch
+    from paper_2608_28511_gb300.layer import MoeLayer
+    D, E, H = 128, 8, 256
+    La = MoeLayer(64, 1, 2, D, E, 64, "bf16", H=H, device="cpu")
+    assert La.latent_fused
+    assert La.w_down.is_contiguous() and La.w_router.is_contiguous()
+    assert La.w_down.data_ptr() == La.w_down_router.data_ptr()
+    assert La.w_router.data_ptr() == La.w_down_router.data_ptr() + D * H * 2
+    assert La.dx_cat.shape == (64, D + E) and La.dx_lat.data_ptr() == La.dx_cat.data_ptr()
+    assert La.dx_lat.stride() == (D + E, 1)
+    for kw in ({"router": "sigmoid"}, {"dtype": "f32"}):
+        args = dict(dtype="bf16", H=H, device="cpu")
+        args.update(kw)
+        Lb = MoeLayer(64, 1, 2, D, E, 64, **args)
+        assert not Lb.latent_fused and Lb.w_down_router is None and Lb.dx_lat.is_contiguous()
+    Lc = MoeLayer(64, 1, 2, D, E, 64, "bf16", device="cpu")
+    assert not Lc.latent_fused and Lc.w_down is None
