@@ -6,7 +6,10 @@ synthetic tokens resident in HBM.  With N GPUs (torchrun) every rank runs its
 own tokens (weak scaling; the layer has no data-path exchange on one node's
 replicas).  Prints one JSON line on rank 0.
 
-    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload C2] [--impl reference]
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload C5] [--impl reference]
+
+The default workload is the largest single-GPU one: skewed routing, T = 32768
+tokens (S = 8192, GBS = 4), D = 2048, E = 128, K = 8, F = 1024.
 """
 from __future__ import annotations
 
@@ -89,6 +92,38 @@ def kernel_work(name: str, w: synth.Workload, T: int, Fs: int = 0, latent_fused:
     return "hbm", float(byts.get(base, 0.0))
 
 
+def gemm_bytes(name: str, w: synth.Workload, T: int, Fs: int = 0, latent_fused: bool = False) -> float:
+    """Algorithmic DRAM bytes of a tensor-core GEMM launch: every operand read
+    once, every result written once (fp32 weight gradients at 4 bytes, an
+    accumulate output read and written).  With the flops this gives the
+    combined roof max(flops / tensor peak, bytes / HBM bandwidth)."""
+    TK, D, E, F, bx = T * w.K, w.D, w.E, w.F, w.b_x
+    Din = w.H if w.H else D
+    base = name.rsplit("_", 1)[0] if name.endswith(("_tc", "_simt")) else name
+    H = w.H
+    table = {
+        "ffn1_swiglu": (TK * D + E * 2 * F * D + TK * 3 * F) * bx,
+        "ffn2": (TK * F + E * D * F + TK * D) * bx,
+        "ffn2_dgrad": (TK * D + E * D * F + TK * F) * bx,
+        "ffn2_wgrad": (TK * F + TK * D) * bx + E * D * F * 4,
+        "ffn1_dgrad": (TK * 2 * F + E * 2 * F * D + TK * D) * bx,
+        "ffn1_wgrad": (TK * 2 * F + TK * D) * bx + E * 2 * F * D * 4,
+        # the two projections (down: x -> x_lat, up: y_lat -> y) move the same bytes
+        "latent_fwd": (T * H + H * D + T * D) * bx,
+        "latent_dgrad": (T * (D + (E if latent_fused else 0)) + (D + (E if latent_fused else 0)) * H + T * H) * bx,
+        "latent_wgrad": (T * H + T * D) * bx + H * D * 4,
+        "router_dgrad": (T * E + E * Din + 2 * T * Din) * bx,
+        "router_wgrad": (T * E + T * Din) * bx + E * Din * 4,
+        "shared_fc1": (T * Din + Fs * Din + 2 * T * Fs) * bx,
+        "shared_fc2": (T * Fs + Din * Fs + 2 * T * Din) * bx,
+        "shared_fc2_dgrad": (T * Din + Din * Fs + T * Fs) * bx,
+        "shared_fc1_dgrad": (T * Fs + Fs * Din + 2 * T * Din) * bx,
+        "shared_fc2_wgrad": (T * Din + T * Fs) * bx + Din * Fs * 4,
+        "shared_fc1_wgrad": (T * Fs + T * Din) * bx + Fs * Din * 4,
+    }
+    return float(table.get(base, 0.0))
+
+
 def expert_flops(w: synth.Workload, T: int) -> float:
     return 18.0 * T * w.K * w.D * w.F
 
@@ -104,32 +139,61 @@ def permute_family_bytes(w: synth.Workload, T: int) -> float:
 # ---------------------------------------------------------------------------
 
 class ClockSampler:
+    """nvidia-smi samples of the SM clock and throttle reasons, read by a
+    thread as they arrive.  ``window()`` brackets a timed region; ``stop()``
+    summarises the samples that arrived inside any window (a sample reports
+    the clock at its own instant, so only those belong to the timed work)."""
     QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
-    def __init__(self, gpu_index: int):
+    def __init__(self, gpu_index: int, interval_ms: int = 20):
+        import threading
         self.proc = None
         self.gpu = gpu_index
+        self.samples = []            # (arrival time, csv line)
+        self.windows = []            # (start, end) of the timed regions
+        self._open = None
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", str(gpu_index), f"--query-gpu={self.QUERY}", "--format=csv,noheader,nounits",
-                 "-lms", "50"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+                 "-lms", str(interval_ms)], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True, bufsize=1)
         except (OSError, ValueError):
             self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+        t0 = time.perf_counter()             # the first sample marks the sampler as running
+        while not self.samples and self.proc.poll() is None and time.perf_counter() - t0 < 5.0:
+            time.sleep(0.01)
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.samples.append((time.perf_counter(), line))
+
+    def begin(self):
+        self._open = time.perf_counter()
+
+    def end(self):
+        if self._open is not None:
+            self.windows.append((self._open, time.perf_counter()))
+            self._open = None
 
     def stop(self):
         if self.proc is None:
             return None
+        time.sleep(0.05)
         self.proc.terminate()
         try:
-            out, _ = self.proc.communicate(timeout=5)
+            self.proc.wait(timeout=5)
         except subprocess.TimeoutExpired:
             self.proc.kill()
-            out, _ = self.proc.communicate()
+            self.proc.wait()
+        self.thread.join(timeout=5)
+        inside = [ln for t, ln in self.samples if any(a <= t <= b for a, b in self.windows)]
         sm, mx, reasons = [], [], set()
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        for line in out.splitlines():
+        for line in inside:
             f = [x.strip() for x in line.split(",")]
             if len(f) < 9:
                 continue
@@ -144,7 +208,10 @@ class ClockSampler:
         if not sm:
             return None
         return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "samples": len(sm),
-                "reasons": sorted(reasons)}
+                "sm_mhz_min": min(sm), "reasons": sorted(reasons),
+                "windows_s": round(sum(b - a for a, b in self.windows), 3),
+                "note": "nvidia-smi every 20 ms; samples inside the device-timed, per-kernel-event and "
+                        "end-to-end passes"}
 
 
 # ---------------------------------------------------------------------------
@@ -279,12 +346,223 @@ def job_throughput(world: int, T: int, t_max_ms: float) -> float:
 # GPU arm
 # ---------------------------------------------------------------------------
 
+def gated_build(world: int, local: int, barrier, build_fn=None) -> None:
+    """Build the library once per node: local rank 0 compiles and links while
+    the other ranks wait at the barrier, then every other rank runs the build
+    too, which finds everything up to date and only loads the library.
+    ``build_fn`` defaults to ``__graft_entry__.build``."""
+    if build_fn is None:
+        import __graft_entry__
+        build_fn = __graft_entry__.build
+    if world > 1 and local != 0:
+        barrier()
+        build_fn()
+        return
+    build_fn()
+    if world > 1:
+        barrier()
+
+
+def kernel_table(prof: dict, steps: int, w: synth.Workload, T: int, Fs: int, latent_fused: bool, peaks: dict):
+    """Per-kernel launches, time, and rate against its roof.  Tensor kernels
+    also get the combined roof max(flops / tensor peak, bytes / HBM) with the
+    bytes counting every operand once and the fp32 weight-gradient writes."""
+    kernels = {}
+    for name, (n, ms) in prof.items():
+        bound, work = kernel_work(name, w, T, Fs, latent_fused)
+        per_launch_ms = ms / max(n, 1)
+        k = {"launches_per_step": n / steps, "ms_per_step": ms / steps, "bound": bound, "work_per_launch": work,
+             "avg_launch_ms": per_launch_ms}
+        if bound == "tensor":
+            k["tflops"] = work / (per_launch_ms * 1e-3) / 1e12
+            k["frac_of_tensor_peak"] = k["tflops"] / peaks["bf16_tflops"]
+            byts = gemm_bytes(name, w, T, Fs, latent_fused)
+            roof_ms = max(work / (peaks["bf16_tflops"] * 1e12), byts / (peaks["hbm_gbs"] * 1e9)) * 1e3
+            k["bytes_per_launch"] = byts
+            k["combined_roof_ms"] = roof_ms
+            k["frac_of_combined_roof"] = roof_ms / per_launch_ms
+            k["roof_bound"] = "tensor" if work / peaks["bf16_tflops"] / 1e12 >= byts / peaks["hbm_gbs"] / 1e9 \
+                else "hbm"
+        else:
+            k["gbs"] = work / (per_launch_ms * 1e-3) / 1e9
+            k["frac_of_hbm"] = k["gbs"] / peaks["hbm_gbs"]
+        kernels[name] = k
+    return kernels
+
+
+def kernel_detail(kernels: dict) -> dict:
+    out = {}
+    for k, v in sorted(kernels.items(), key=lambda kv: -kv[1]["ms_per_step"]):
+        d = {"ms_per_step": round(v["ms_per_step"], 4)}
+        if v["bound"] == "tensor":
+            d.update({"TFLOP/s": round(v["tflops"], 1), "frac": round(v["frac_of_tensor_peak"], 3),
+                      "combined_roof_frac": round(v["frac_of_combined_roof"], 3), "roof_bound": v["roof_bound"]})
+        else:
+            d.update({"GB/s": round(v["gbs"], 1), "frac": round(v["frac_of_hbm"], 3)})
+        out[k] = d
+    return out
+
+
+def top_roofline(kernels: dict, w: synth.Workload, peaks: dict) -> dict:
+    """Roofline of the kernel with the largest share of the step.  Kernels run
+    inside a step of a few milliseconds, so a contraction's fraction is taken
+    of the burst bf16 peak; the sustained (seconds-long) figure rides along."""
+    tname, tk = max(kernels.items(), key=lambda kv: kv[1]["ms_per_step"])
+    traffic = None
+    tpath = os.path.join(ROOT, "profiles", "traffic.json")
+    if os.path.exists(tpath):
+        with open(tpath) as f:
+            tr = json.load(f)
+        ent = tr.get(w.name, {}).get(tname)
+        if ent is not None:
+            import hashlib
+            src = os.path.join(ROOT, ent["src"])
+            sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16] if os.path.exists(src) else None
+            traffic = ent["bytes"] if sha == ent["sha256_16"] else None   # stale once the kernel changed
+    if tk["bound"] == "tensor":
+        achieved = tk["tflops"]
+        return {"kernel": tname, "bound": "tensor", "achieved": achieved, "peak": peaks["bf16_tflops"],
+                "unit": "TFLOP/s", "frac": achieved / peaks["bf16_tflops"], "traffic": traffic,
+                "peak_note": f"bf16 dense, burst, of {peaks['source']}",
+                "peak_sustained": peaks["bf16_tflops_sustained"],
+                "frac_sustained": achieved / peaks["bf16_tflops_sustained"],
+                "algorithmic_bytes": tk["bytes_per_launch"], "frac_of_combined_roof": tk["frac_of_combined_roof"],
+                "launch_ms": tk["avg_launch_ms"]}
+    achieved = tk["gbs"]
+    return {"kernel": tname, "bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+            "frac": achieved / peaks["hbm_gbs"], "traffic": traffic, "peak_note": f"HBM copy, of {peaks['source']}",
+            "launch_ms": tk["avg_launch_ms"]}
+
+
+def measure(w: synth.Workload, args, rank: int, world: int, barrier, clocks=None, e2e_steps: int = 0,
+            steps: int | None = None, router: str = "softmax", shared_width: int = 0, payload: str = "bf16"):
+    """Build one layer of workload ``w`` (this rank's seeded tokens), warm it
+    up, capture its step as a CUDA graph and time ``steps`` steps twice: once
+    with only per-step events (the headline), once with events around every
+    kernel (per-kernel rooflines).  With ``e2e_steps`` also time the public
+    host-buffer call.  Returns the measurements; frees the layer."""
+    import torch
+    from paper_2608_28511_gb300 import abi
+    from paper_2608_28511_gb300.layer import MoeLayer
+
+    steps = args.steps if steps is None else steps
+    T = w.T
+    inputs = synth.make_inputs(w, seed=rank_seed(w, rank))      # each rank its own tokens
+    if router == "sigmoid":
+        inputs["expert_bias"] = synth.make_expert_bias(w.E, rank_seed(w, rank))
+    if shared_width:
+        inputs.update(synth.make_shared_expert(w, shared_width, rank_seed(w, rank)))
+    L = MoeLayer(w.S, w.GBS, w.K, w.D, w.E, w.F, w.dtype, w.H, router=router, shared_F=shared_width,
+                 payload=payload)
+    L.load(inputs)
+    stream = torch.cuda.current_stream()
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device="cuda")
+
+    for _ in range(args.warmup):
+        L.step()
+    torch.cuda.synchronize()
+    assert abi.moe_check_device_status() == 0
+
+    graph = None
+    if not args.no_graph:
+        graph = L.capture()          # the step's launches, replayed as one graph
+        graph.replay()
+        torch.cuda.synchronize()
+
+    def timed_steps(kernel_events: bool):
+        """``steps`` steps, L2 flushed before each (outside the step events).
+        With kernel_events the library also brackets every kernel with CUDA
+        events on its stream (per-kernel durations for the roofline); those
+        records sit between the kernels, so the headline step time comes from
+        the pass without them."""
+        ev_s = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
+        ev_e = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
+        abi.moe_prof_reset()
+        abi.moe_prof_enable(kernel_events)
+        n0 = abi.moe_launch_count()
+        barrier()
+        torch.cuda.synchronize()
+        if clocks is not None:
+            clocks.begin()
+        t0 = time.perf_counter()
+        use_graph = graph is not None and not kernel_events
+        for i in range(steps):
+            flush.zero_()
+            ev_s[i].record(stream)
+            if use_graph:
+                graph.replay()
+            else:
+                L.step()
+            ev_e[i].record(stream)
+        torch.cuda.synchronize()
+        if clocks is not None:
+            clocks.end()
+        barrier()
+        wall = time.perf_counter() - t0
+        launches = (abi.moe_launch_count() - n0) // steps
+        abi.moe_prof_enable(False)
+        prof = abi.moe_prof_read() if kernel_events else {}
+        per_step = [s.elapsed_time(e) for s, e in zip(ev_s, ev_e)]
+        return per_step, wall, launches, prof
+
+    per_step, wall, _, _ = timed_steps(kernel_events=False)
+    step_ms = sum(per_step) / len(per_step)
+    t_max = max_over_ranks(step_ms, world, "cuda")
+    assert abi.moe_check_device_status() == 0
+    per_step_ev, _, launches, prof = timed_steps(kernel_events=True)
+    assert abi.moe_check_device_status() == 0
+
+    # ---- end to end through the public API with host buffers
+    e2e = None
+    if e2e_steps > 0:
+        x_h = inputs["x"].pin_memory()
+        dy_h = inputs["dy"].pin_memory()
+        y_h = torch.empty_like(x_h).pin_memory()
+        dx_h = torch.empty_like(x_h).pin_memory()
+        h2d = x_h.numel() * x_h.element_size() + dy_h.numel() * dy_h.element_size()
+        d2h = y_h.numel() * y_h.element_size() + dx_h.numel() * dx_h.element_size()
+        # the public host-batch call: every step's x and dy copied in and its y
+        # and dx copied out inside the timed region, overlapped with the
+        # neighbouring steps' compute (two device buffer sets, two copy streams)
+        L.prepare_host_pipeline(graphs=graph is not None)
+        batch = (x_h, dy_h, y_h, dx_h)
+        L.run_host([batch] * 2)
+        torch.cuda.synchronize()
+        e_s, e_e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        barrier()
+        if clocks is not None:
+            clocks.begin()
+        e_s.record(stream)
+        L.run_host([batch] * e2e_steps)
+        e_e.record(stream)
+        torch.cuda.synchronize()
+        if clocks is not None:
+            clocks.end()
+        e2e_ms = max_over_ranks(e_s.elapsed_time(e_e) / e2e_steps, world, "cuda")
+        e2e = {"value": job_throughput(world, T, e2e_ms), "unit": UNIT, "h2d_bytes_per_step": h2d,
+               "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms, "steps": e2e_steps,
+               "api": "MoeLayer.run_host: step i+1's H2D and step i's D2H on two copy streams, overlapping compute"}
+    out = {"T": T, "step_ms": step_ms, "t_max": t_max, "per_step": per_step, "wall": wall,
+           "step_ms_ev": sum(per_step_ev) / len(per_step_ev), "launches": launches, "prof": prof, "e2e": e2e,
+           "latent_fused": L.latent_fused, "graph": graph is not None}
+    del graph, L, flush, inputs
+    torch.cuda.synchronize()
+    torch.cuda.empty_cache()
+    return out
+
+
 def main() -> None:
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--steps", type=int, default=50)
     ap.add_argument("--warmup", type=int, default=5)
-    ap.add_argument("--workload", default="C2")
+    ap.add_argument("--workload", default="C5",
+                    help="C1..C5 or a workload name; default C5, the largest single-GPU workload (skewed routing, "
+                         "T = 32768, E = 128, K = 8)")
+    ap.add_argument("--per-workload", default="C2,C3,C4",
+                    help="other workloads timed after the headline one (device-timed step and per-kernel "
+                         "fractions, 1 GPU only; empty = none)")
+    ap.add_argument("--per-workload-steps", type=int, default=20)
     ap.add_argument("--seed", type=int, default=None,
                     help="input seed of rank 0 (default: the workload's own, 0); seeds 1 and 2 give the variance check")
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
@@ -322,149 +600,43 @@ def main() -> None:
         dist.init_process_group("nccl")
     torch.cuda.set_device(local)
 
-    import __graft_entry__
-    __graft_entry__.build()
-    from paper_2608_28511_gb300 import abi
-    from paper_2608_28511_gb300.layer import MoeLayer
-
-    T = w.T
-    inputs = synth.make_inputs(w, seed=rank_seed(w, rank))      # each rank its own tokens
-    if args.router == "sigmoid":
-        inputs["expert_bias"] = synth.make_expert_bias(w.E, rank_seed(w, rank))
-    if args.shared_width:
-        inputs.update(synth.make_shared_expert(w, args.shared_width, rank_seed(w, rank)))
-    L = MoeLayer(w.S, w.GBS, w.K, w.D, w.E, w.F, w.dtype, w.H, router=args.router, shared_F=args.shared_width,
-                 payload=args.payload)
-    L.load(inputs)
-    stream = torch.cuda.current_stream()
-    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device="cuda")
-
     def barrier():
         if world > 1:
             dist.barrier()
 
-    for _ in range(args.warmup):
-        L.step()
-    torch.cuda.synchronize()
-    assert abi.moe_check_device_status() == 0
+    gated_build(world, local, barrier)
+    from paper_2608_28511_gb300 import abi  # noqa: F401
 
-    graph = None
-    if not args.no_graph:
-        graph = L.capture()          # the step's launches, replayed as one graph
-        graph.replay()
-        torch.cuda.synchronize()
-
-    def timed_steps(kernel_events: bool):
-        """K steps, L2 flushed before each (outside the step events).  With
-        kernel_events the library also brackets every kernel with CUDA events
-        on its stream (per-kernel durations for the roofline); those records
-        sit between the kernels, so the headline step time comes from the pass
-        without them."""
-        ev_s = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
-        ev_e = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
-        abi.moe_prof_reset()
-        abi.moe_prof_enable(kernel_events)
-        n0 = abi.moe_launch_count()
-        barrier()
-        torch.cuda.synchronize()
-        t0 = time.perf_counter()
-        use_graph = graph is not None and not kernel_events
-        for i in range(args.steps):
-            flush.zero_()
-            ev_s[i].record(stream)
-            if use_graph:
-                graph.replay()
-            else:
-                L.step()
-            ev_e[i].record(stream)
-        torch.cuda.synchronize()
-        barrier()
-        wall = time.perf_counter() - t0
-        launches = (abi.moe_launch_count() - n0) // args.steps
-        abi.moe_prof_enable(False)
-        prof = abi.moe_prof_read() if kernel_events else {}
-        per_step = [s.elapsed_time(e) for s, e in zip(ev_s, ev_e)]
-        return per_step, wall, launches, prof
-
-    clocks = ClockSampler(local)
-    per_step, wall, _, _ = timed_steps(kernel_events=False)
-    clk = clocks.stop()
-    step_ms = sum(per_step) / len(per_step)
-    step_stats = step_statistics(per_step)
-    t_max = max_over_ranks(step_ms, world, "cuda")
-    assert abi.moe_check_device_status() == 0
-    per_step_ev, _, launches, prof = timed_steps(kernel_events=True)
-    step_ms_ev = sum(per_step_ev) / len(per_step_ev)
-    assert abi.moe_check_device_status() == 0
-
-    # ---- end to end through the public API with host buffers
-    e2e = None
-    if args.e2e_steps > 0:
-        x_h = inputs["x"].pin_memory()
-        dy_h = inputs["dy"].pin_memory()
-        y_h = torch.empty_like(x_h).pin_memory()
-        dx_h = torch.empty_like(x_h).pin_memory()
-        h2d = x_h.numel() * x_h.element_size() + dy_h.numel() * dy_h.element_size()
-        d2h = y_h.numel() * y_h.element_size() + dx_h.numel() * dx_h.element_size()
-        # the public host-batch call: every step's x and dy copied in and its y
-        # and dx copied out inside the timed region, overlapped with the
-        # neighbouring steps' compute (two device buffer sets, two copy streams)
-        L.prepare_host_pipeline(graphs=graph is not None)
-        batch = (x_h, dy_h, y_h, dx_h)
-        L.run_host([batch] * 2)
-        torch.cuda.synchronize()
-        e_s, e_e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        barrier()
-        e_s.record(stream)
-        L.run_host([batch] * args.e2e_steps)
-        e_e.record(stream)
-        torch.cuda.synchronize()
-        e2e_ms = max_over_ranks(e_s.elapsed_time(e_e) / args.e2e_steps, world, "cuda")
-        e2e = {"value": job_throughput(world, T, e2e_ms), "unit": UNIT, "h2d_bytes_per_step": h2d,
-               "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms, "steps": args.e2e_steps,
-               "api": "MoeLayer.run_host: step i+1's H2D and step i's D2H on two copy streams, overlapping compute"}
-
-    # ---- per-kernel roofline from the live events
     peaks = _peaks()
-    kernels = {}
-    for name, (n, ms) in prof.items():
-        bound, work = kernel_work(name, w, T, args.shared_width, L.latent_fused)
-        per_launch_ms = ms / max(n, 1)
-        kernels[name] = {"launches_per_step": n / args.steps, "ms_per_step": ms / args.steps,
-                         "bound": bound, "work_per_launch": work, "avg_launch_ms": per_launch_ms}
-    top = max(kernels.items(), key=lambda kv: kv[1]["ms_per_step"])
-    tname, tk = top
-    traffic = None
-    tpath = os.path.join(ROOT, "profiles", "traffic.json")
-    if os.path.exists(tpath):
-        with open(tpath) as f:
-            tr = json.load(f)
-        ent = tr.get(w.name, {}).get(tname)
-        if ent is not None:
-            import hashlib
-            src = os.path.join(ROOT, ent["src"])
-            sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16] if os.path.exists(src) else None
-            traffic = ent["bytes"] if sha == ent["sha256_16"] else None   # stale once the kernel changed
-    if tk["bound"] == "tensor":
-        achieved = tk["work_per_launch"] / (tk["avg_launch_ms"] * 1e-3) / 1e12
-        peak = peaks["bf16_tflops_sustained"]
-        roof = {"kernel": tname, "bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
-                "frac": achieved / peak, "traffic": traffic,
-                "peak_note": f"bf16 dense, sustained, of {peaks['source']}"}
-    else:
-        achieved = tk["work_per_launch"] / (tk["avg_launch_ms"] * 1e-3) / 1e9
-        peak = peaks["hbm_gbs"]
-        roof = {"kernel": tname, "bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                "frac": achieved / peak, "traffic": traffic, "peak_note": f"HBM copy, of {peaks['source']}"}
+    clocks = ClockSampler(local)
+    r = measure(w, args, rank, world, barrier, clocks=clocks, e2e_steps=args.e2e_steps, router=args.router,
+                shared_width=args.shared_width, payload=args.payload)
+    clk = clocks.stop()
+    T = r["T"]
+    kernels = kernel_table(r["prof"], args.steps, w, T, args.shared_width, r["latent_fused"], peaks)
+    roof = top_roofline(kernels, w, peaks)
 
     exp_ms = sum(v["ms_per_step"] for k, v in kernels.items() if k.startswith("ffn") or k == "swiglu_bwd")
     perm_names = ("dispatch_rows", "combine", "combine_bwd", "dispatch_bwd", "dispatch_route_bwd")
     perm_ms = sum(v["ms_per_step"] for k, v in kernels.items() if k in perm_names)
-    detail = {k: {"ms_per_step": round(v["ms_per_step"], 4),
-                  ("TFLOP/s" if v["bound"] == "tensor" else "GB/s"):
-                      round(v["work_per_launch"] / (v["avg_launch_ms"] * 1e-3) / (1e12 if v["bound"] == "tensor"
-                                                                                   else 1e9), 1)}
-              for k, v in sorted(kernels.items(), key=lambda kv: -kv[1]["ms_per_step"])}
+
+    # ---- the other workloads, device-timed only (1 GPU)
+    per_workload = None
+    names = [n for n in args.per_workload.split(",") if n.strip()] if world == 1 else []
+    if names:
+        per_workload = {}
+        for n in names:
+            wn = synth.get(n.strip())
+            if wn.name == w.name:
+                continue
+            rn = measure(wn, args, rank, world, barrier, steps=args.per_workload_steps)
+            kn = kernel_table(rn["prof"], args.per_workload_steps, wn, wn.T, 0, rn["latent_fused"], peaks)
+            top = top_roofline(kn, wn, peaks)
+            per_workload[wn.name] = {
+                "ms_per_step": round(rn["step_ms"], 4), "tokens_per_s": wn.T / (rn["step_ms"] * 1e-3),
+                "steps": args.per_workload_steps, "step_stats": step_statistics(rn["per_step"]),
+                "top_kernel": {k: top[k] for k in ("kernel", "bound", "achieved", "unit", "frac")},
+                "kernels": kernel_detail(kn)}
 
     cpu = None
     if (rank == 0 and world == 1 and not args.no_cpu_baseline and args.router == "softmax" and not args.shared_width
@@ -472,6 +644,7 @@ def main() -> None:
         cpu = cpu_baseline(w, args.cpu_budget)
 
     if rank == 0:
+        t_max = r["t_max"]
         line = {
             "metric": METRIC, "value": job_throughput(world, T, t_max), "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": t_max, "higher_is_better": True,
@@ -480,21 +653,22 @@ def main() -> None:
                        "H": w.H, "seed": w.seed, "router": args.router, "shared_width": args.shared_width,
                        "payload": args.payload,
                        "parallelism": f"replicas x{world}, each rank its own tokens",
-                       "launch": "one CUDA graph per step" if graph is not None else "eager launches",
+                       "launch": "one CUDA graph per step" if r["graph"] else "eager launches",
                        "l2": "256 MiB buffer written before every timed step (outside the step events); "
-                             "the step also touches ~3 GB > 129 MB L2"},
+                             "the step also touches several GB > 129 MB L2"},
             "roofline": roof,
             "dispatch_gbs": permute_family_bytes(w, T) / (perm_ms * 1e-3) / 1e9 if perm_ms else None,
             "expert_tflops": expert_flops(w, T) / (exp_ms * 1e-3) / 1e12 if exp_ms else None,
             "cpu_baseline": cpu,
-            "e2e": e2e,
-            "gpu_launches": launches * args.steps,
-            "gpu_launches_per_step": launches,
+            "e2e": r["e2e"],
+            "gpu_launches": r["launches"] * args.steps,
+            "gpu_launches_per_step": r["launches"],
             "clocks": clk,
-            "wall_s_timed_region": wall,
-            "ms_per_step_kernel_events_pass": round(step_ms_ev, 4),
-            "step_stats": step_stats,
-            "kernels": detail,
+            "wall_s_timed_region": r["wall"],
+            "ms_per_step_kernel_events_pass": round(r["step_ms_ev"], 4),
+            "step_stats": step_statistics(r["per_step"]),
+            "kernels": kernel_detail(kernels),
+            "per_workload": per_workload,
         }
         print(json.dumps(line), flush=True)
     if world > 1:

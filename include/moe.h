@@ -172,8 +172,13 @@ int moe_dequant_nvfp4(const moe_shape_t* shape, const void* x_perm_q, const uint
  *  - A shape whose table does not fit (E * ceil(T*K / 2048) > 262144) returns
  *    MOE_ERR_TOO_LARGE before anything is enqueued.
  *  - The first call on a device looks up that device's copy of the array
- *    (cudaGetSymbolAddress, with the device current); make that first call
- *    before any stream capture on the device.
+ *    (cudaGetSymbolAddress, with the device current).  With CUDA's lazy module
+ *    loading that first lookup is also when the library's module is loaded on
+ *    the device and the array is placed, which may allocate device memory and
+ *    synchronise; only the calls after it allocate nothing.  Make one warm-up
+ *    call per device at initialisation, before any stream capture.
+ *  - On a device with an ordinal of 64 or more the call returns MOE_ERR_CUDA
+ *    (cudaErrorInvalidDevice) without enqueuing anything.
  *  - All calls share the one array.  Each call writes every table entry it
  *    reads before reading it, so nothing from an earlier call leaks into a
  *    result; but calls whose kernels overlap on the GPU (different streams or

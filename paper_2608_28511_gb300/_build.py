@@ -3,7 +3,10 @@
 Each ``csrc/*.cu`` translation unit compiles in parallel to an object under
 ``_build/``; the objects link into ``paper_2608_28511_gb300/libmoe.so`` with the
 CUDA runtime linked statically.  A unit is recompiled only when it or a header
-is newer than its object.
+is newer than its object.  Objects and the library are written under
+per-process temporary names and renamed into place, so two processes that
+build at once never leave a half-written file; callers that run one process
+per GPU still build on one rank and let the others wait (bench.py).
 """
 from __future__ import annotations
 
@@ -41,24 +44,36 @@ def _headers_mtime() -> float:
 
 
 def _compile(nvcc: str, src: str, obj: str, extra: list[str]) -> str:
-    cmd = [nvcc] + NVCC_FLAGS + extra + ["-c", src, "-o", obj]
+    tmp = f"{obj}.{os.getpid()}.tmp"
+    cmd = [nvcc] + NVCC_FLAGS + extra + ["-c", src, "-o", tmp]
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError(f"nvcc failed for {os.path.basename(src)}:\n{r.stdout}\n{r.stderr}")
+    os.replace(tmp, obj)
     return r.stderr
 
 
-def build(verbose: bool = False, force: bool = False, extra_flags: list[str] | None = None) -> str:
-    """Compile every CUDA source and link libmoe.so.  Returns the library path."""
+# sources compiled by the last build() call of this process
+last_compiled: list[str] = []
+
+
+def build(verbose: bool = False, force: bool = False, extra_flags: list[str] | None = None,
+          csrc: str | None = None, build_dir: str | None = None, lib: str | None = None) -> str:
+    """Compile every CUDA source and link libmoe.so.  Returns the library path.
+    ``csrc``, ``build_dir`` and ``lib`` default to the package's own sources,
+    ``_build/<machine>`` and ``libmoe.so``."""
+    csrc = csrc or CSRC
+    build_dir = build_dir or BUILD
+    lib = lib or LIB
     nvcc = _nvcc()
-    os.makedirs(BUILD, exist_ok=True)
+    os.makedirs(build_dir, exist_ok=True)
     extra = list(extra_flags or [])
-    srcs = sorted(glob.glob(os.path.join(CSRC, "*.cu")))
+    srcs = sorted(glob.glob(os.path.join(csrc, "*.cu")))
     hdr_t = _headers_mtime()
     jobs = []
     objs = []
     for s in srcs:
-        o = os.path.join(BUILD, os.path.basename(s)[:-3] + ".o")
+        o = os.path.join(build_dir, os.path.basename(s)[:-3] + ".o")
         objs.append(o)
         if force or not os.path.exists(o) or os.path.getmtime(o) < max(os.path.getmtime(s), hdr_t):
             jobs.append((s, o))
@@ -69,15 +84,16 @@ def build(verbose: bool = False, force: bool = False, extra_flags: list[str] | N
                 msg = f.result()
                 if verbose and msg.strip():
                     print(f"[{os.path.basename(futs[f])}]\n{msg}", file=sys.stderr)
+    last_compiled[:] = [s for s, _ in jobs]
     newest = max(os.path.getmtime(o) for o in objs)
-    if force or jobs or not os.path.exists(LIB) or os.path.getmtime(LIB) < newest:
-        tmp = LIB + ".tmp"
+    if force or jobs or not os.path.exists(lib) or os.path.getmtime(lib) < newest:
+        tmp = f"{lib}.{os.getpid()}.tmp"
         cmd = [nvcc] + ARCH + ["-shared", "-o", tmp] + objs
         r = subprocess.run(cmd, capture_output=True, text=True)
         if r.returncode != 0:
             raise RuntimeError(f"link failed:\n{r.stdout}\n{r.stderr}")
-        os.replace(tmp, LIB)
-    return LIB
+        os.replace(tmp, lib)
+    return lib
 
 
 if __name__ == "__main__":

@@ -5,9 +5,10 @@
 // that has already reserved all device memory for its own pool, a step loop
 // that forbids allocation, or a runtime that cannot afford cudaMalloc's
 // implicit device-wide synchronisation.  For them the counting sort's scratch
-// (per-chunk expert histograms and their prefix sums) lives in a fixed array
-// compiled into the library: every GPU that loads the library holds one copy
-// of it until the process exits.  The call allocates nothing.
+// (the per-chunk expert histogram table) lives in a fixed array compiled into
+// the library: every GPU that loads the library holds one copy of it until the
+// process exits.  After the first call on a device (which loads this module
+// there and looks up the array's address) the call allocates nothing.
 #include <mutex>
 
 #include "common.cuh"
@@ -15,7 +16,8 @@
 
 namespace moe {
 
-// Scratch of the counting sort: 2 * E * ceil(T*K / 2048) int32 values.
+// Scratch of the counting sort: E * ceil(T*K / 2048) int32 per-chunk counts
+// (counts[e * nchunks + chunk]).
 static __device__ __align__(256) int32_t g_dispatch_scratch[MOE_DISPATCH_NOALLOC_SCRATCH_INTS];
 
 namespace {
@@ -28,6 +30,7 @@ int32_t* g_scratch_ptr[kMaxDevices] = {};
 // g_dispatch_scratch is only a host-side stand-in, so the address is looked up
 // once per device, with that device current, and passed to the kernels.
 int scratch_for_device(int dev, int32_t** out) {
+  if (dev < 0 || dev >= kMaxDevices) return abi_cuda_status(cudaErrorInvalidDevice);
   std::lock_guard<std::mutex> lk(g_scratch_mu);
   if (!g_scratch_ptr[dev]) {
     void* p = nullptr;

@@ -67,26 +67,24 @@ __device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
 __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
 }
-// CL: acquire at cluster scope (barriers that the other CTA of a pair signals).
-template <bool CL = false>
+// Waits on barriers that the other CTA of a pair signals (the leader's full and
+// accumulator-empty barriers) use the default CTA scope too.  What crosses CTAs
+// there is either asynchronous-proxy completion (TMA complete_tx, tcgen05.commit),
+// whose mbarrier completion already makes the data visible to the waiter, or a
+// pure write-after-read hand-off of TMEM: an epilogue thread arrives only after
+// tcgen05.wait::ld has returned its loads into registers and
+// tcgen05.fence::before_thread_sync has ordered them before the arrive, so the
+// MMA that then overwrites the accumulator cannot change what was read.  No
+// generic-proxy data is published through these barriers.
 __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
   uint32_t ok;
-  if (CL)
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-        "selp.u32 %0, 1, 0, p;\n\t}\n"
-        : "=r"(ok)
-        : "r"(bar), "r"(parity)
-        : "memory");
-  else
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-        "selp.u32 %0, 1, 0, p;\n\t}\n"
-        : "=r"(ok)
-        : "r"(bar), "r"(parity)
-        : "memory");
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}\n"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
   return ok != 0;
 }
 __device__ __forceinline__ uint64_t global_timer_ns() {
@@ -95,13 +93,12 @@ __device__ __forceinline__ uint64_t global_timer_ns() {
   return t;
 }
 // Wait for phase `parity` of `bar`; false if the CTA aborted or the limit expired.
-template <bool CL = false>
 __device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, volatile int* abort_flag,
                                              uint32_t* err) {
-  if (mbar_try_wait<CL>(bar, parity)) return true;
+  if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = global_timer_ns();
   for (uint32_t i = 1;; ++i) {
-    if (mbar_try_wait<CL>(bar, parity)) return true;
+    if (mbar_try_wait(bar, parity)) return true;
     if ((i & 63u) == 0) {
       if (*abort_flag) return false;
       if (global_timer_ns() - t0 > kWaitLimitNs) {
@@ -113,10 +110,9 @@ __device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, vola
   }
 }
 // Same, ignoring the abort flag (used while draining).
-template <bool CL = false>
 __device__ __forceinline__ bool wait_drain(uint32_t bar, uint32_t parity, uint64_t limit_ns) {
   const uint64_t t0 = global_timer_ns();
-  while (!mbar_try_wait<CL>(bar, parity)) {
+  while (!mbar_try_wait(bar, parity)) {
     if (global_timer_ns() - t0 > limit_ns) return false;
   }
   return true;
@@ -588,7 +584,7 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
       }
       for (int kb = 0; kb < ti.nkb; ++kb) {
         int okw = 1;
-        if (lane == 0) okw = wait_bounded<CG == 2>(smem_u32(&empty[stage]), phase ^ 1u, &s_abort, p.err) ? 1 : 0;
+        if (lane == 0) okw = wait_bounded(smem_u32(&empty[stage]), phase ^ 1u, &s_abort, p.err) ? 1 : 0;
         okw = __shfl_sync(0xffffffffu, okw, 0);
         if (!okw) { ok = false; break; }
         const uint32_t fb_local = smem_u32(&full[stage]);
@@ -660,7 +656,7 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
       int s = stage;
       uint32_t ph = phase;
       for (int i = 0; i < C::kStages; ++i) {
-        wait_drain<CG == 2>(smem_u32(&empty[s]), ph ^ 1u, 1000000000ull);
+        wait_drain(smem_u32(&empty[s]), ph ^ 1u, 1000000000ull);
         if (++s == C::kStages) { s = 0; ph ^= 1u; }
       }
     }
@@ -668,7 +664,7 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
       const int pending = issued < C::kStages ? issued : C::kStages;
       for (int i = 0; i < pending; ++i) {
         stage = (stage + C::kStages - 1) % C::kStages;
-        wait_drain<CG == 2>(smem_u32(&full[stage]), (last_phase >> stage) & 1u, 1000000000ull);
+        wait_drain(smem_u32(&full[stage]), (last_phase >> stage) & 1u, 1000000000ull);
       }
     }
   } else if (warp == 0) {
@@ -684,7 +680,7 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
         decode_tile<GROUP, CG>(p, t, s_off, s_pref, rank, ti);
         const int64_t nb = ti.n0 * BN + (int64_t)rank * BNC;  // this CTA's first B row / column
         for (int kb = 0; kb < ti.nkb; ++kb) {
-          if (!wait_bounded<CG == 2>(smem_u32(&empty[stage]), phase ^ 1u, &s_abort, p.err)) { ok = false; break; }
+          if (!wait_bounded(smem_u32(&empty[stage]), phase ^ 1u, &s_abort, p.err)) { ok = false; break; }
           const uint32_t fb_local = smem_u32(&full[stage]);
           // CG 2: both CTAs' copies complete on the leader's barrier, which expects both
           const uint32_t fb = CG == 2 ? map_to_rank(fb_local, 0) : fb_local;
@@ -741,7 +737,7 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
         int s = stage;
         uint32_t ph = phase;
         for (int i = 0; i < C::kStages; ++i) {
-          wait_drain<CG == 2>(smem_u32(&empty[s]), ph ^ 1u, 1000000000ull);
+          wait_drain(smem_u32(&empty[s]), ph ^ 1u, 1000000000ull);
           if (++s == C::kStages) { s = 0; ph ^= 1u; }
         }
       }
@@ -751,7 +747,7 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
         const int pending = issued < C::kStages ? issued : C::kStages;
         for (int i = 0; i < pending; ++i) {
           stage = (stage + C::kStages - 1) % C::kStages;
-          wait_drain<CG == 2>(smem_u32(&full[stage]), (last_phase >> stage) & 1u, 1000000000ull);
+          wait_drain(smem_u32(&full[stage]), (last_phase >> stage) & 1u, 1000000000ull);
         }
       }
     }
@@ -769,11 +765,11 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
       decode_tile<GROUP, CG>(p, t, s_off, s_pref, rank, ti);
       if (ti.nkb == 0) continue;
       issued_any = true;
-      if (!wait_bounded<CG == 2>(smem_u32(&tempty[acc]), acc_phase ^ 1u, &s_abort, p.err)) { ok = false; break; }
+      if (!wait_bounded(smem_u32(&tempty[acc]), acc_phase ^ 1u, &s_abort, p.err)) { ok = false; break; }
       tc_fence_after();
       const uint32_t d_tmem = tmem_base + (uint32_t)(acc * BN);
       for (int kb = 0; kb < ti.nkb; ++kb) {
-        if (!wait_bounded<CG == 2>(smem_u32(&full[stage]), phase, &s_abort, p.err)) { ok = false; break; }
+        if (!wait_bounded(smem_u32(&full[stage]), phase, &s_abort, p.err)) { ok = false; break; }
         tc_fence_after();
         const uint32_t sa = smem_u32(smem + stage * C::kStageBytes);
         const uint32_t sb = sa + C::kABytes;
@@ -800,7 +796,7 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
     // drain: all MMAs issued by this warp have completed before TMEM is freed
     if (lane == 0 && issued_any) {
       mma_commit_cg<CG>(smem_u32(done), 0x1);
-      wait_drain<CG == 2>(smem_u32(done), 0, 1000000000ull);
+      wait_drain(smem_u32(done), 0, 1000000000ull);
     }
     __syncwarp();
   } else {
@@ -861,7 +857,7 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
         for (int i = 0; i < kPre; ++i)
           if (ch + i * CSTEP < nch_acc) acc_fetch(c_rows, ldc_b, n0 + (ch + i * CSTEP) * 32, lane, nrows, pre[i]);
       }
-      if (!wait_bounded<CG == 2>(smem_u32(&tfull[acc]), acc_phase, &s_abort, p.err)) break;
+      if (!wait_bounded(smem_u32(&tfull[acc]), acc_phase, &s_abort, p.err)) break;
       tc_fence_after();
       const uint32_t tbase = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
       float v[32];

@@ -100,3 +100,58 @@ def test_every_timed_kernel_has_algorithmic_work():
     missing = [n for n in sorted(names - no_work) if bench.kernel_work(n, w, w.T, 2688)[1] <= 0]
     assert not missing, missing
     assert len(names) >= 30
+
+
+_TINY_CU = 'extern "C" __global__ void tiny_kernel(int* p) { p[threadIdx.x] = 1; }\n' \
+           'extern "C" int tiny_version(void) { return 7; }\n'
+
+
+def _build_worker(rank, world, port, root, q):
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), RANK=str(rank), WORLD_SIZE=str(world),
+                      LOCAL_RANK=str(rank))
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        import functools
+        from paper_2608_28511_gb300 import _build
+        fn = functools.partial(_build.build, csrc=os.path.join(root, "csrc"), build_dir=os.path.join(root, "obj"),
+                               lib=os.path.join(root, "libtiny.so"))
+        bench.gated_build(world, rank, dist.barrier, build_fn=fn)
+        dist.barrier()
+        q.put((rank, [os.path.basename(s) for s in _build.last_compiled]))
+    finally:
+        dist.destroy_process_group()
+
+
+def test_gated_build_compiles_stale_objects_once_per_node(tmp_path):
+    """Two ranks start a build over an object older than its source: local rank
+    0 recompiles and links while rank 1 waits, then rank 1 finds everything up
+    to date.  No temporary file is left behind."""
+    import shutil
+    import time
+    if shutil.which("nvcc") is None and not os.path.exists("/usr/local/cuda/bin/nvcc"):
+        pytest.skip("nvcc not available")
+    from paper_2608_28511_gb300 import _build
+    root = str(tmp_path)
+    os.makedirs(os.path.join(root, "csrc"))
+    src = os.path.join(root, "csrc", "tiny.cu")
+    with open(src, "w") as f:
+        f.write(_TINY_CU)
+    lib = os.path.join(root, "libtiny.so")
+    _build.build(csrc=os.path.join(root, "csrc"), build_dir=os.path.join(root, "obj"), lib=lib)
+    time.sleep(1.1)
+    os.utime(src)                                  # the object is now stale
+    world = 2
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_build_worker, args=(r, world, port, root, q)) for r in range(world)]
+    for p in procs:
+        p.start()
+    for p in procs:
+        p.join(timeout=300)
+        assert p.exitcode == 0
+    res = dict(q.get(timeout=10) for _ in range(world))
+    assert res[0] == ["tiny.cu"]                  # rank 0 rebuilt the stale unit
+    assert res[1] == []                            # rank 1 found it fresh
+    assert os.path.getmtime(os.path.join(root, "obj", "tiny.o")) >= os.path.getmtime(src)
+    assert not [n for n in os.listdir(root) + os.listdir(os.path.join(root, "obj")) if n.endswith(".tmp")]
