@@ -304,6 +304,17 @@ int moe_route_sigmoid(const moe_shape_t* shape, const void* x, const void* w_rou
                       float aux_coef, float* logits, int32_t* topk_idx, float* topk_prob, float* aux_f,
                       float* aux_loss, void* ws, size_t ws_bytes, void* stream);
 
+/* The selection and balance-statistics stage of moe_route_sigmoid on given
+ * fp32 logits [T, E] (Sec. 5.2; readings S1-S3): topk_idx, topk_prob, aux_f
+ * and aux_loss exactly as moe_route_sigmoid computes them from its own
+ * logits.  select_keys [T, E] fp32 (optional, NULL = not written) receives
+ * every key the selection compared, s + expert_bias with s = sigmoid(logits),
+ * formed by the same fp32 arithmetic: the K largest of a row, ties to the
+ * lower expert, are topk_idx.  Workspace as moe_route_sigmoid. */
+int moe_topk_sigmoid(const moe_shape_t* shape, const float* logits, const float* expert_bias, float aux_coef,
+                     float* select_keys, int32_t* topk_idx, float* topk_prob, float* aux_f, float* aux_loss,
+                     void* ws, size_t ws_bytes, void* stream);
+
 /* Sigmoid router backward: gradient of (the downstream loss through
  * topk_prob, given as dtopk_prob [T, K]) + aux_grad * aux_loss with respect to
  * the logits, with aux_f from moe_route_sigmoid (a count: no gradient) and

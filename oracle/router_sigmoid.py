@@ -24,23 +24,42 @@ import numpy as np
 
 from .moe import sigmoid
 
-__all__ = ["sigmoid_route", "seq_aux_loss", "sigmoid_route_bwd"]
+__all__ = ["sigmoid_route", "seq_aux_loss", "sigmoid_route_bwd", "select_on_keys"]
 
 
-def sigmoid_route(z: np.ndarray, K: int, expert_bias=None, idx_override=None):
+def select_on_keys(keys: np.ndarray, K: int) -> np.ndarray:
+    """Reading S1's choice on given selection keys [T, E]: per token the K
+    largest keys, ties to the lower expert index, best first.  Given the fp32
+    keys s + b that the GPU formed, this is the stage-isolated choice its
+    indices must equal bit for bit (the keys' own rounding is then the same
+    on both sides)."""
+    T, E = keys.shape
+    idx = np.empty((T, K), dtype=np.int64)
+    for t in range(T):
+        row = [float(v) for v in keys[t]]
+        idx[t] = sorted(range(E), key=lambda e: (-row[e], e))[:K]
+    return idx
+
+
+def sigmoid_route(z: np.ndarray, K: int, expert_bias=None, idx_override=None, keys=None):
     """Readings S1, S2.  Returns idx [T, K] int64 and prob [T, K] float64.
 
     ``idx_override`` replaces the choice (where a near-tie of s + b could
     resolve either way); the gate values are then S2 over the given set.
+    ``keys`` [T, E] chooses on those selection keys (``select_on_keys``)
+    instead of the float64 s + b.
     """
     T, E = z.shape
     s = sigmoid(z)
     b = np.zeros(E) if expert_bias is None else np.asarray(expert_bias, dtype=np.float64)
     idx = np.empty((T, K), dtype=np.int64)
     prob = np.empty((T, K))
+    chosen_on_keys = select_on_keys(keys, K) if keys is not None and idx_override is None else None
     for t in range(T):
         if idx_override is not None:
             chosen = [int(e) for e in idx_override[t]]
+        elif chosen_on_keys is not None:
+            chosen = [int(e) for e in chosen_on_keys[t]]
         else:
             key = [s[t, e] + b[e] for e in range(E)]
             chosen = sorted(range(E), key=lambda e: (-key[e], e))[:K]

@@ -35,7 +35,7 @@ EXPORTS = (
     "moe_ce_composition", "moe_ce_layer_pattern", "moe_route_sigmoid", "moe_route_sigmoid_bwd",
     "moe_shared_expert", "moe_shared_expert_bwd", "moe_expert_ffn_gather", "moe_expert_ffn_bwd_gather",
     "moe_dispatch_fp8", "moe_dequant_rows", "moe_dispatch_nvfp4", "moe_dequant_nvfp4", "moe_dispatch_route_bwd",
-    "moe_latent_route_bwd",
+    "moe_latent_route_bwd", "moe_topk_sigmoid",
 )
 
 
@@ -89,6 +89,7 @@ _SIGS = {
     "moe_dispatch_route_bwd": ([_SHP] + [_VP] * 12 + [_SZ, _VP], ctypes.c_int),
     "moe_latent_route_bwd": ([_SHP] + [_VP] * 14 + [_SZ, _VP], ctypes.c_int),
     "moe_route_sigmoid": ([_SHP, _VP, _VP, _VP, _F32, _VP, _VP, _VP, _VP, _VP, _VP, _SZ, _VP], ctypes.c_int),
+    "moe_topk_sigmoid": ([_SHP, _VP, _VP, _F32, _VP, _VP, _VP, _VP, _VP, _VP, _SZ, _VP], ctypes.c_int),
     "moe_route_sigmoid_bwd": ([_SHP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _F32, _F32, _VP, _VP, _VP, _VP, _SZ, _VP],
                               ctypes.c_int),
     "moe_expert_ffn_gather": ([_SHP] + [_VP] * 9 + [_SZ, _VP], ctypes.c_int),
@@ -302,6 +303,13 @@ def moe_route_sigmoid(shape, x, w_router, expert_bias, aux_coef, logits, topk_id
     _check("moe_route_sigmoid", lib().moe_route_sigmoid(
         _shape(shape), _p(x), _p(w_router), _p(expert_bias), float(aux_coef), _p(logits), _p(topk_idx),
         _p(topk_prob), _p(aux_f), _p(aux_loss), _p(ws), _nbytes(ws), _stream(stream)))
+
+
+def moe_topk_sigmoid(shape, logits, expert_bias, aux_coef, select_keys, topk_idx, topk_prob, aux_f, aux_loss, ws,
+                     stream=None):
+    _check("moe_topk_sigmoid", lib().moe_topk_sigmoid(
+        _shape(shape), _p(logits), _p(expert_bias), float(aux_coef), _p(select_keys), _p(topk_idx), _p(topk_prob),
+        _p(aux_f), _p(aux_loss), _p(ws), _nbytes(ws), _stream(stream)))
 
 
 def moe_route_sigmoid_bwd(shape, x, w_router, logits, topk_idx, topk_prob, dtopk_prob, aux_f, aux_coef, aux_grad,

@@ -996,6 +996,28 @@ int moe_route_sigmoid(const moe_shape_t* shape, const void* x, const void* w_rou
   return MOE_OK;
 }
 
+int moe_topk_sigmoid(const moe_shape_t* shape, const float* logits, const float* expert_bias, float aux_coef,
+                     float* select_keys, int32_t* topk_idx, float* topk_prob, float* aux_f, float* aux_loss, void* ws,
+                     size_t ws_bytes, void* stream) {
+  Dims d;
+  TRY(check_shape(shape, &d));
+  REQUIRE_PTR(logits);
+  OPTIONAL_PTR(expert_bias);
+  OPTIONAL_PTR(select_keys);
+  REQUIRE_PTR(topk_idx);
+  REQUIRE_PTR(topk_prob);
+  REQUIRE_PTR(aux_f);
+  REQUIRE_PTR(aux_loss);
+  REQUIRE_PTR(ws);
+  if (ws_bytes < ws_route_sigmoid(d)) return MOE_ERR_WORKSPACE;
+  if (!(aux_coef == aux_coef)) return MOE_ERR_SHAPE;
+  Ctx c;
+  TRY(get_ctx(stream, &c));
+  TRY_CUDA(launch_route_sigmoid_select(c, logits, expert_bias, d.T, d.S, d.GBS, d.E, d.K, aux_coef, topk_idx,
+                                       topk_prob, aux_f, aux_loss, ws, select_keys));
+  return MOE_OK;
+}
+
 int moe_route_sigmoid_bwd(const moe_shape_t* shape, const void* x, const void* w_router, const float* logits,
                           const int32_t* topk_idx, const float* topk_prob, const float* dtopk_prob,
                           const float* aux_f, float aux_coef, float aux_grad, void* dx, float* dw_router,

@@ -67,7 +67,7 @@ size_t route_sigmoid_fwd_ws_bytes(int64_t T, int64_t S, int64_t GBS, int E);
 // balance loss.
 cudaError_t launch_route_sigmoid_select(const Ctx& c, const float* logits, const float* bias, int64_t T, int64_t S,
                                         int64_t GBS, int E, int K, float coef, int32_t* idx, float* prob,
-                                        float* f_out, float* loss, void* ws);
+                                        float* f_out, float* loss, void* ws, float* keys = nullptr);
 // dz [T, E] fp32 (fully written) and optionally a bf16 copy.
 cudaError_t launch_route_dz_sigmoid(const Ctx& c, const float* logits, const int32_t* idx, const float* prob,
                                     const float* dprob, const float* f, int64_t T, int64_t S, int64_t GBS, int E,

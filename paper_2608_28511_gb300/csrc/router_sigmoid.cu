@@ -31,12 +31,14 @@ struct SigmoidOp {
 // tokens, chooses each token's K experts by s + b (four threads per token),
 // writes idx and the gate values s_k / sum over the chosen of s, then adds up,
 // per expert, the normalised scores (in token order) and the choice counts of
-// its tokens: one partial per (sequence, chunk).
+// its tokens: one partial per (sequence, chunk).  With `keys` the block also
+// writes every selection key s + b it compared, formed by the same fp32
+// addition of the same staged operands as in the selection.
 template <int KM>
 __global__ void __launch_bounds__(256) select_sigmoid_kernel(
     const float* __restrict__ logits, const float* __restrict__ bias, int64_t S, int E, int K, int tpb, int nch,
     int32_t* __restrict__ idx, float* __restrict__ prob, float* __restrict__ psum, int32_t* __restrict__ pcnt,
-    uint32_t* __restrict__ ticket) {
+    uint32_t* __restrict__ ticket, float* __restrict__ keys) {
   extern __shared__ __align__(16) float sm[];
   float* zs = sm;                                   // [tpb][E] scores
   float* bs = zs + tpb * E;                         // [E]
@@ -52,6 +54,10 @@ __global__ void __launch_bounds__(256) select_sigmoid_kernel(
   }
   if (ch == 0 && g == 0 && tid == 0) *ticket = 0u;  // for the finalize kernel that follows
   __syncthreads();
+  if (keys) {
+    float* kout = keys + t0 * E;
+    for (int i = tid; i < n * E; i += blockDim.x) kout[i] = __fadd_rn(zs[i], bs[i % E]);
+  }
   const int q = tid >> 2, r = tid & 3;
   const bool active = q < n;
   const float* row = zs + (int64_t)q * E;
@@ -239,7 +245,7 @@ size_t route_sigmoid_fwd_ws_bytes(int64_t T, int64_t S, int64_t GBS, int E) {
 
 cudaError_t launch_route_sigmoid_select(const Ctx& c, const float* logits, const float* bias, int64_t T, int64_t S,
                                         int64_t GBS, int E, int K, float coef, int32_t* idx, float* prob,
-                                        float* f_out, float* loss, void* ws) {
+                                        float* f_out, float* loss, void* ws, float* keys) {
   if (T == 0) return cudaSuccess;
   const int tpb = sel::tokens_per_block(E);
   const int64_t nch = select_chunks(S, E);
@@ -256,7 +262,7 @@ cudaError_t launch_route_sigmoid_select(const Ctx& c, const float* logits, const
     KernelScope ks("select_sigmoid", c.stream);
 #define MOE_SELECT_SIGMOID(KM)                                                                             \
   select_sigmoid_kernel<KM><<<grid, 4 * tpb, smem, c.stream>>>(logits, bias, S, E, K, tpb, (int)nch, idx, \
-                                                               prob, psum, pcnt, ticket)
+                                                               prob, psum, pcnt, ticket, keys)
     switch (sel::k_bound(K)) {
       case 2: MOE_SELECT_SIGMOID(2); break;
       case 4: MOE_SELECT_SIGMOID(4); break;

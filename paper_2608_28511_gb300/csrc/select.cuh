@@ -99,7 +99,7 @@ __device__ __forceinline__ void quad_topk(const float* __restrict__ row, const f
     const float vn = (active && cn < E) ? row[cn] : 0.f;  // next column, loaded ahead
     if (active && c < E) {
       sum += v;
-      const uint64_t p = pack(bias ? v + bias[c] : v, c);
+      const uint64_t p = pack(bias ? __fadd_rn(v, bias[c]) : v, c);
       if (p > L[KM - 1]) {
         uint64_t cv = p;
 #pragma unroll

@@ -40,13 +40,18 @@ def test_sigmoid_router_full_size():
     torch.cuda.synchronize()
     z = f64(L.logits)
     bias = inp["expert_bias"].double().numpy()
-    idx_ref, _ = O.sigmoid_route(z, W.K, bias)
     idx = i64(L.topk_idx)
-    keys = O.sigmoid(z) + bias[None, :]
-    top = -np.sort(-keys, axis=1)[:, : W.K + 1]
-    ties = set(np.nonzero((top[:, :-1] - top[:, 1:] < 1e-6).any(axis=1))[0].tolist())
-    differ = set(np.nonzero((idx != idx_ref).any(axis=1))[0].tolist())
-    assert differ <= ties
+    # the selection kernel's own fp32 keys s + b: the choice is bitwise on every token
+    from paper_2608_28511_gb300 import abi
+    keys_t = torch.empty_like(L.logits)
+    idx_t = torch.empty_like(L.topk_idx)
+    abi.moe_topk_sigmoid(L.shape, L.logits, L.expert_bias, L.aux_coef, keys_t, idx_t, torch.empty_like(L.topk_prob),
+                         torch.empty_like(L.aux_f), torch.empty_like(L.aux_loss), L.ws)
+    torch.cuda.synchronize()
+    keys = f64(keys_t)
+    assert np.array_equal(i64(idx_t), idx)
+    assert np.array_equal(idx, O.select_on_keys(keys, W.K))
+    assert np.abs(keys - (O.sigmoid(z) + bias[None, :])).max() <= 2e-6
     _, prob_at = O.sigmoid_route(z, W.K, bias, idx_override=idx)
     assert np.abs(f64(L.topk_prob) - prob_at).max() <= 1e-5
     loss_ref, f_ref, _ = O.seq_aux_loss(z, idx, W.S, W.GBS, L.aux_coef)

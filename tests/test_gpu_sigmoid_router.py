@@ -1,10 +1,12 @@
 """GPU parity of the sigmoid router (sigmoid scores, selection-only expert
 bias, sequence-level balance loss; Sec. 5.2) against the float64 oracle.
 
-Stage-isolated checks feed the oracle the GPU's own logits, so the choice of
-experts is compared bit for bit except on tokens whose selection keys s + b
-are within 1e-6 of each other (there an fp32 sigmoid may legitimately resolve
-the tie either way; the GPU's choice must then still be a valid top-K).
+Stage-isolated checks feed the oracle the GPU's own fp32 selection keys
+s + b (exported by moe_topk_sigmoid from the selection kernel itself), so the
+choice of experts is compared bit for bit on every token, exact ties included
+(ties go to the lower expert).  From the raw inputs the oracle's float64 keys
+may order two keys that lie within fp32 rounding of each other the other way;
+the end-to-end test allows exactly those tokens and checks the rest bitwise.
 Float results: gate values 1e-5 absolute, balance loss 1e-5 relative, logit
 gradients 1e-4 relative Frobenius (fp32 arithmetic throughout), and the
 router's weight and input gradients 1e-2 relative Frobenius (bf16 GEMMs).
@@ -64,13 +66,43 @@ def run(name, aux_coef=COEF, aux_grad=1.0):
 
 
 def key_tie_tokens(z, bias, K):
-    """Tokens where two of the K+1 largest keys s + b lie within KEY_TIE."""
+    """Tokens where two of the K+1 largest float64 keys s + b lie within KEY_TIE."""
     keys = O.sigmoid(z) + bias[None, :]
     top = -np.sort(-keys, axis=1)[:, : min(K + 1, keys.shape[1])]
     return set(np.nonzero((top[:, :-1] - top[:, 1:] < KEY_TIE).any(axis=1))[0].tolist())
 
 
-def check_choice(idx_gpu, idx_ref, z, bias, K):
+def gpu_keys(L, logits=None, bias="layer"):
+    """Re-run the selection stage on the layer's logits with the key export:
+    (keys [T, E] f64, idx [T, K]) exactly as the selection kernel formed and chose them."""
+    from paper_2608_28511_gb300 import abi
+    logits = L.logits if logits is None else logits
+    b = L.expert_bias if isinstance(bias, str) else bias
+    keys = torch.empty_like(logits)
+    idx = torch.empty(logits.shape[0], L.K, dtype=torch.int32, device=logits.device)
+    prob = torch.empty(logits.shape[0], L.K, dtype=torch.float32, device=logits.device)
+    f = torch.empty_like(L.aux_f)
+    loss = torch.empty_like(L.aux_loss)
+    abi.moe_topk_sigmoid(L.shape, logits, b, L.aux_coef, keys, idx, prob, f, loss, L.ws)
+    torch.cuda.synchronize()
+    return f64(keys), i64(idx), f64(prob), f64(f), float(loss[0].item())
+
+
+def check_choice_bitwise(L, z, bias, K):
+    """The layer's indices equal the oracle's choice on the kernel's own keys,
+    on every token; the keys are sigmoid(z) + b within fp32 rounding."""
+    keys, idx_k, _, _, _ = gpu_keys(L)
+    idx = i64(L.topk_idx)
+    assert np.array_equal(idx_k, idx)                     # the export does not change the choice
+    assert np.array_equal(idx, O.select_on_keys(keys, K))
+    assert np.abs(keys - (O.sigmoid(z) + bias[None, :])).max() <= 2e-6
+    return keys
+
+
+def check_choice_from_raw(idx_gpu, idx_ref, z, bias, K):
+    """From float64 keys of the raw inputs: equal except where two of the K+1
+    largest keys lie within fp32 rounding (KEY_TIE); there the GPU's choice
+    must still be a valid top-K of the float64 keys up to that gap."""
     ties = key_tie_tokens(z, bias, K)
     keys = O.sigmoid(z) + bias[None, :]
     for t in np.nonzero((idx_gpu != idx_ref).any(axis=1))[0]:
@@ -91,10 +123,10 @@ def test_sigmoid_route_stage(name):
     z = f64(L.logits)
     assert rel_frob(z, z_ref) <= LOGIT_REL
     bias = o["expert_bias"]
-    idx_ref, prob_ref = O.sigmoid_route(z, w.K, bias)
+    keys = check_choice_bitwise(L, z, bias, w.K)
     idx = i64(L.topk_idx)
-    check_choice(idx, idx_ref, z, bias, w.K)
-    _, prob_at = O.sigmoid_route(z, w.K, bias, idx_override=idx)
+    idx_ref, prob_at = O.sigmoid_route(z, w.K, bias, keys=keys)
+    assert np.array_equal(idx, idx_ref)
     prob = f64(L.topk_prob)
     assert np.abs(prob - prob_at).max() <= PROB_ABS
     assert np.abs(prob.sum(axis=1) - 1.0).max() <= 1e-6
@@ -157,7 +189,8 @@ def test_sigmoid_layer_end_to_end(name):
     z = O.router_logits(x, wr)
     idx_ref, _ = O.sigmoid_route(z, w.K, o["expert_bias"])
     idx = i64(L.topk_idx)
-    check_choice(idx, idx_ref, z, o["expert_bias"], w.K)
+    check_choice_bitwise(L, f64(L.logits), o["expert_bias"], w.K)
+    check_choice_from_raw(idx, idx_ref, z, o["expert_bias"], w.K)
     idx_use, prob = O.sigmoid_route(z, w.K, o["expert_bias"], idx_override=idx)
     x_in = O.latent_project(x, o["w_down"]) if w.H else x
     off, ros, tor = O.expert_permutation(idx_use, w.E)
@@ -233,3 +266,42 @@ def test_sigmoid_status_errors():
         abi.moe_route_sigmoid(L.shape, L.x, L.w_router, L.expert_bias, COEF, L.logits, L.topk_idx, L.topk_prob,
                               None, L.aux_loss, L.ws)
     assert e.value.status == -4
+
+
+TIE_CASES = [(128, 2, 16, 4), (96, 1, 8, 2), (64, 2, 200, 8), (100, 3, 24, 16)]
+
+
+@pytest.mark.parametrize("S,GBS,E,K", TIE_CASES)
+def test_exact_key_ties_go_to_the_lower_expert(S, GBS, E, K):
+    """Integer logits in [-2, 2] and a bias of a few equal values: most tokens
+    have exactly equal keys at the K-th place.  The kernel's choice equals the
+    oracle's on its exported keys and on the float64 keys (equal (z, b) pairs
+    give equal keys in both precisions; distinct pairs stay far apart), and
+    its gate values and balance statistics match the oracle's."""
+    from paper_2608_28511_gb300 import abi
+    from paper_2608_28511_gb300.layer import MoeLayer
+    T = S * GBS
+    g = torch.Generator().manual_seed(S + E + K)
+    z = torch.randint(-2, 3, (T, E), generator=g).to(torch.float32)
+    bias = (torch.randint(0, 2, (E,), generator=g).to(torch.float32) * 0.25)
+    L = MoeLayer(S, GBS, K, 64, E, 64, "bf16", router="sigmoid")
+    zd, bd = z.cuda(), bias.cuda()
+    keys, idx, prob, f, loss = gpu_keys(L, logits=zd, bias=bd)
+    zf, bf = z.double().numpy(), bias.double().numpy()
+    k64 = O.sigmoid(zf) + bf[None, :]
+    tied = sum(int(np.sort(k64[t])[::-1][K - 1] == np.sort(k64[t])[::-1][K]) for t in range(T)) if K < E else 0
+    assert K == E or tied > T // 4                              # the case really is tie-heavy
+    assert np.array_equal(idx, O.select_on_keys(keys, K))
+    idx_ref, prob_ref = O.sigmoid_route(zf, K, bf)
+    assert np.array_equal(idx, idx_ref)
+    assert np.abs(prob - prob_ref).max() <= PROB_ABS
+    loss_ref, f_ref, _ = O.seq_aux_loss(zf, idx_ref, S, GBS, L.aux_coef)
+    assert np.array_equal(f, f_ref.astype(np.float32).astype(np.float64))
+    assert abs(loss - loss_ref) <= 1e-5 * abs(loss_ref)
+    # the selection stage alone equals the full router on the same logits
+    idx2 = torch.empty(T, K, dtype=torch.int32, device="cuda")
+    prob2 = torch.empty(T, K, dtype=torch.float32, device="cuda")
+    abi.moe_topk_sigmoid(L.shape, zd, bd, L.aux_coef, None, idx2, prob2, L.aux_f, L.aux_loss, L.ws)
+    torch.cuda.synchronize()
+    assert np.array_equal(i64(idx2), idx)
+    assert np.array_equal(f64(prob2), prob)

@@ -244,3 +244,27 @@ def test_nvfp4_payload_mistakes_are_caught(monkeypatch):
     monkeypatch.setattr(N, "nvfp4_quantize_rows", row_amax_scales)
     monkeypatch.setattr(oracle, "nvfp4_quantize_rows", row_amax_scales)
     _expect_failure(PN.test_round_trip_and_bf16_exactness)
+
+
+def test_sigmoid_key_selection_mistakes_are_caught(monkeypatch):
+    import oracle.router_sigmoid as RS
+    import tests.test_oracle_sigmoid as PS
+
+    def ties_to_higher(keys, K):
+        T, E = keys.shape
+        return np.array([sorted(range(E), key=lambda e: (-float(keys[t, e]), -e))[:K] for t in range(T)],
+                        dtype=np.int64)
+
+    monkeypatch.setattr(RS, "select_on_keys", ties_to_higher)
+    monkeypatch.setattr(oracle, "select_on_keys", ties_to_higher)
+    _expect_failure(PS.test_selection_on_given_keys_against_brute_force_with_exact_ties, 8, 3)
+    _expect_failure(PS.test_gates_on_key_choice_use_scores_not_keys)
+
+    def ascending(keys, K):
+        T, E = keys.shape
+        return np.array([sorted(range(E), key=lambda e: (-float(keys[t, e]), e))[:K][::-1] for t in range(T)],
+                        dtype=np.int64)
+
+    monkeypatch.setattr(RS, "select_on_keys", ascending)
+    monkeypatch.setattr(oracle, "select_on_keys", ascending)
+    _expect_failure(PS.test_selection_on_given_keys_against_brute_force_with_exact_ties, 8, 3)

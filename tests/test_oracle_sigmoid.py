@@ -112,3 +112,37 @@ def test_router_gradient_matches_central_differences():
             assert abs(fd - dz[i, j]) <= 1e-7 * max(1.0, abs(fd)), (i, j, fd, dz[i, j])
     np.testing.assert_allclose(dxr, dz @ w, rtol=1e-13)
     np.testing.assert_allclose(dwr, dz.T @ x, rtol=1e-13)
+
+
+@pytest.mark.parametrize("E,K", [(6, 2), (8, 3), (5, 5), (9, 4)])
+def test_selection_on_given_keys_against_brute_force_with_exact_ties(E, K):
+    """select_on_keys: the unique K-set that beats every other expert (larger
+    key, or an equal key and a lower index), ordered best first; integer keys
+    with many exact ties exercise the tie rule."""
+    keys = _rng(40 + E).integers(-2, 3, size=(60, E)).astype(np.float32)
+    idx = O.select_on_keys(keys, K)
+    for t in range(60):
+        assert set(idx[t].tolist()) == _winners(keys[t].astype(np.float64), K)
+        k = keys[t, idx[t]]
+        assert all(k[j] > k[j + 1] or (k[j] == k[j + 1] and idx[t, j] < idx[t, j + 1]) for j in range(K - 1))
+
+
+def test_selection_on_keys_matches_the_float64_route_when_keys_are_its_own():
+    r = _rng(41)
+    z = r.normal(size=(40, 10)) * 2
+    b = r.normal(size=10) * 0.2
+    keys = scipy.special.expit(z) + b[None, :]
+    idx_keys, prob_keys = O.sigmoid_route(z, 3, b, keys=keys)
+    idx, prob = O.sigmoid_route(z, 3, b)
+    assert (idx_keys == idx).all()
+    np.testing.assert_array_equal(prob_keys, prob)
+
+
+def test_gates_on_key_choice_use_scores_not_keys():
+    # equal keys from different (score, bias) pairs: the choice is by key, the gates by score
+    z = np.array([[0.0, np.log(3.0), 0.0]])         # s = 0.5, 0.75, 0.5
+    b = np.array([0.25, 0.0, -0.5])                 # keys 0.75, 0.75, 0.0
+    keys = scipy.special.expit(z) + b[None, :]
+    idx, prob = O.sigmoid_route(z, 2, b, keys=keys)
+    assert idx.tolist() == [[0, 1]]                 # tie at 0.75 -> lower expert first
+    np.testing.assert_allclose(prob[0], [0.5 / 1.25, 0.75 / 1.25], rtol=1e-15)
