@@ -15,7 +15,8 @@ import torch
 
 import oracle as O
 import synth
-from tests.gpu_util import LOGIT_REL, PROB_ABS, REL_FROB, f64, i64, make_layer, oracle_inputs, rel_frob
+from tests.gpu_util import (LOGIT_REL, PROB_ABS, REL_FROB, assert_close, f64, i64, make_layer, oracle_inputs,
+                            rel_frob)
 
 pytestmark = pytest.mark.gpu
 
@@ -83,10 +84,10 @@ def test_expert_ffn_stage(name):
     w, L, inp, o = run(name)
     g, u, a, y = O.expert_ffn(f64(L.x_perm), i64(L.expert_offsets), o["w_gate"], o["w_up"], o["w2"])
     hg, hu = L.unpack_h(L.h)
-    assert rel_frob(f64(hg), g) <= REL_FROB
-    assert rel_frob(f64(hu), u) <= REL_FROB
-    assert rel_frob(f64(L.act), a) <= REL_FROB
-    assert rel_frob(f64(L.y_perm), y) <= REL_FROB
+    assert_close(f64(hg), g, what='f64(hg)')
+    assert_close(f64(hu), u, what='f64(hu)')
+    assert_close(f64(L.act), a, what='f64(L.act)')
+    assert_close(f64(L.y_perm), y, what='f64(L.y_perm)')
 
 
 @pytest.mark.parametrize("name", names)
@@ -94,10 +95,10 @@ def test_combine_stage(name):
     w, L, inp, o = run(name)
     y = O.combine(f64(L.y_perm), f64(L.prob_perm), i64(L.row_of_slot), w.T, w.K)
     y_gpu = L.y_lat if w.H else L.y
-    assert rel_frob(f64(y_gpu), y) <= REL_FROB
+    assert_close(f64(y_gpu), y, what='f64(y_gpu)')
     if w.H:
-        assert rel_frob(f64(L.y), O.latent_project(f64(L.y_lat), o["w_upp"])) <= REL_FROB
-        assert rel_frob(f64(L.x_lat), O.latent_project(o["x"], o["w_down"])) <= REL_FROB
+        assert_close(f64(L.y), O.latent_project(f64(L.y_lat), o["w_upp"]), what='f64(L.y)')
+        assert_close(f64(L.x_lat), O.latent_project(o["x"], o["w_down"]), what='f64(L.x_lat)')
 
 
 @pytest.mark.parametrize("name", names)
@@ -105,12 +106,12 @@ def test_combine_bwd_stage(name):
     w, L, inp, o = run(name)
     dy = f64(L.dy_lat) if w.H else o["dy"]
     dyp, dpp = O.combine_bwd(dy, f64(L.y_perm), f64(L.prob_perm), i64(L.token_of_row))
-    assert rel_frob(f64(L.dy_perm), dyp) <= REL_FROB
-    assert rel_frob(f64(L.dprob_perm), dpp) <= REL_FROB
+    assert_close(f64(L.dy_perm), dyp, what='f64(L.dy_perm)')
+    assert_close(f64(L.dprob_perm), dpp, what='f64(L.dprob_perm)')
     if w.H:
         dyl, dwu = O.latent_project_bwd(o["dy"], f64(L.y_lat), o["w_upp"])
-        assert rel_frob(f64(L.dy_lat), dyl) <= REL_FROB
-        assert rel_frob(f64(L.dw_upp), dwu) <= REL_FROB
+        assert_close(f64(L.dy_lat), dyl, what='f64(L.dy_lat)')
+        assert_close(f64(L.dw_upp), dwu, what='f64(L.dw_upp)')
 
 
 @pytest.mark.parametrize("name", names)
@@ -120,10 +121,10 @@ def test_expert_ffn_bwd_stage(name):
     dxp, dwg, dwu, dw2 = O.expert_ffn_bwd(f64(L.dy_perm), f64(L.x_perm), f64(hg), f64(hu), i64(L.expert_offsets),
                                           o["w_gate"], o["w_up"], o["w2"])
     gg, gu = L.unpack_w1_like(L.dw1)
-    assert rel_frob(f64(L.dx_perm), dxp) <= REL_FROB
-    assert rel_frob(f64(gg), dwg) <= REL_FROB
-    assert rel_frob(f64(gu), dwu) <= REL_FROB
-    assert rel_frob(f64(L.dw2), dw2) <= REL_FROB
+    assert_close(f64(L.dx_perm), dxp, what='f64(L.dx_perm)')
+    assert_close(f64(gg), dwg, rows=1, what='f64(gg)')
+    assert_close(f64(gu), dwu, rows=1, what='f64(gu)')
+    assert_close(f64(L.dw2), dw2, rows=1, what='f64(L.dw2)')
     # experts with no rows get exactly zero weight gradients
     cnt = np.diff(i64(L.expert_offsets))
     for e in np.nonzero(cnt == 0)[0]:
@@ -136,15 +137,15 @@ def test_dispatch_and_route_bwd_stage(name):
     dx_e, dprob = O.dispatch_bwd(f64(L.dx_perm), f64(L.dprob_perm), i64(L.row_of_slot), w.T, w.K)
     assert np.array_equal(f64(L.dprob), dprob)                     # a pure gather of fp32 values
     dz, dx_r, dw_r = O.route_bwd(o["x"], o["w_router"], i64(L.topk_idx), f64(L.topk_prob), f64(L.dprob))
-    assert rel_frob(f64(L.dlogits), dz) <= REL_FROB
-    assert rel_frob(f64(L.dw_router), dw_r) <= REL_FROB
+    assert_close(f64(L.dlogits), dz, what='f64(L.dlogits)')
+    assert_close(f64(L.dw_router), dw_r, rows=1, what='f64(L.dw_router)')
     if w.H:
-        assert rel_frob(f64(L.dx_lat), dx_e) <= REL_FROB
+        assert_close(f64(L.dx_lat), dx_e, what='f64(L.dx_lat)')
         dx_h, dw_down = O.latent_project_bwd(f64(L.dx_lat), o["x"], o["w_down"])
-        assert rel_frob(f64(L.dw_down), dw_down) <= REL_FROB
-        assert rel_frob(f64(L.dx), dx_h + dx_r) <= REL_FROB
+        assert_close(f64(L.dw_down), dw_down, what='f64(L.dw_down)')
+        assert_close(f64(L.dx), dx_h + dx_r, what='f64(L.dx)')
     else:
-        assert rel_frob(f64(L.dx), dx_e + dx_r) <= REL_FROB
+        assert_close(f64(L.dx), dx_e + dx_r, what='f64(L.dx)')
     # I5: dz rows sum to zero
     assert np.abs(f64(L.dlogits).sum(axis=1)).max() <= 1e-5 * max(1.0, np.abs(dz).max())
 
@@ -163,18 +164,21 @@ def test_end_to_end(name):
                           idx_override=idx_gpu, **kw)
     bwd = O.layer_backward(fwd, o["dy"], o["x"], o["w_router"], o["w_gate"], o["w_up"], o["w2"], **kw)
     assert np.abs(f64(L.topk_prob) - fwd["prob"]).max() <= PROB_ABS
-    assert rel_frob(f64(L.y), fwd["y"]) <= REL_FROB
-    assert rel_frob(f64(L.dx), bwd["dx"]) <= REL_FROB
+    assert_close(f64(L.y), fwd["y"], what='f64(L.y)')
+    assert_close(f64(L.dx), bwd["dx"], what='f64(L.dx)')
     gg, gu = L.unpack_w1_like(L.dw1)
-    assert rel_frob(f64(gg), bwd["dw_gate"]) <= REL_FROB
-    assert rel_frob(f64(gu), bwd["dw_up"]) <= REL_FROB
-    assert rel_frob(f64(L.dw2), bwd["dw2"]) <= REL_FROB
+    assert_close(f64(gg), bwd["dw_gate"], rows=1, what='f64(gg)')
+    assert_close(f64(gu), bwd["dw_up"], rows=1, what='f64(gu)')
+    assert_close(f64(L.dw2), bwd["dw2"], rows=1, what='f64(L.dw2)')
+    # end to end a rarely chosen expert's router row sums a few dz values that
+    # cancel, so the router weight gradient is checked as a whole here (per
+    # expert in the stage test, from the GPU's own dprob)
     assert rel_frob(f64(L.dw_router), bwd["dw_router"]) <= REL_FROB
-    assert rel_frob(f64(L.dlogits), bwd["dz"]) <= REL_FROB
-    assert rel_frob(f64(L.dprob), bwd["dprob"]) <= REL_FROB
+    assert_close(f64(L.dlogits), bwd["dz"], what='f64(L.dlogits)')
+    assert_close(f64(L.dprob), bwd["dprob"], what='f64(L.dprob)')
     if w.H:
-        assert rel_frob(f64(L.dw_down), bwd["dw_down"]) <= REL_FROB
-        assert rel_frob(f64(L.dw_upp), bwd["dw_upp"]) <= REL_FROB
+        assert_close(f64(L.dw_down), bwd["dw_down"], what='f64(L.dw_down)')
+        assert_close(f64(L.dw_upp), bwd["dw_upp"], what='f64(L.dw_upp)')
 
 
 # ---------------------------------------------------------------------------
@@ -201,11 +205,14 @@ def test_edge_shapes_end_to_end(w):
     assert (i64(L.expert_offsets) == off).all() and (i64(L.row_of_slot) == ros).all()
     fwd = O.layer_forward(o["x"], o["w_router"], o["w_gate"], o["w_up"], o["w2"], w.K, idx_override=idx_gpu)
     bwd = O.layer_backward(fwd, o["dy"], o["x"], o["w_router"], o["w_gate"], o["w_up"], o["w2"])
-    assert rel_frob(f64(L.y), fwd["y"]) <= REL_FROB
-    assert rel_frob(f64(L.dx), bwd["dx"]) <= REL_FROB
-    assert rel_frob(f64(L.dw2), bwd["dw2"]) <= REL_FROB
+    assert_close(f64(L.y), fwd["y"], what='f64(L.y)')
+    assert_close(f64(L.dx), bwd["dx"], what='f64(L.dx)')
+    assert_close(f64(L.dw2), bwd["dw2"], rows=1, what='f64(L.dw2)')
     gg, gu = L.unpack_w1_like(L.dw1)
-    assert rel_frob(f64(gg), bwd["dw_gate"]) <= REL_FROB
+    assert_close(f64(gg), bwd["dw_gate"], rows=1, what='f64(gg)')
+    # end to end a rarely chosen expert's router row sums a few dz values that
+    # cancel, so the router weight gradient is checked as a whole here (per
+    # expert in the stage test, from the GPU's own dprob)
     assert rel_frob(f64(L.dw_router), bwd["dw_router"]) <= REL_FROB
 
 
@@ -220,7 +227,7 @@ def test_all_tokens_on_one_expert():
     assert (i64(L.token_of_row) == np.arange(300)).all()
     o = oracle_inputs(inp)
     fwd = O.layer_forward(o["x"], o["w_router"], o["w_gate"], o["w_up"], o["w2"], 1, bias=o["bias"])
-    assert rel_frob(f64(L.y), fwd["y"]) <= REL_FROB
+    assert_close(f64(L.y), fwd["y"], what='f64(L.y)')
     for e in (0, 1, 7):
         assert float(L.dw2[e].abs().max()) == 0.0
 
