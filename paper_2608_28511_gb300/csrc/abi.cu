@@ -837,7 +837,8 @@ static int router_grad_gemms(const Ctx& c, const Dims& d, const void* x, const v
   if (dgrad && d.T > 0) TRY_CUDA(gemm(c, a, "router_dgrad_tc", "router_dgrad_simt"));
   const int splits = d.dt == DType::BF16 ? router_splits(d, c.num_sms) : 1;
   if (splits > 1) {
-    // split-K: partial products of equal token ranges, then their in-order sum
+    // split-K: partial products of token ranges of near-equal size that start
+    // on 64-row boundaries, then their in-order sum
     GemmDesc bs = b;
     bs.group = Group::K;
     bs.num_groups = splits;

@@ -269,17 +269,18 @@ cudaError_t launch_gemm_tc(const Ctx& c, const GemmDesc& d, const char* name) {
     const tc::TailTemplates* tails = tail_templates(d.A, a_inner, pl.lda * 2, gb ? nullptr : d.B, b_inner, pl.ldb * 2);
     if (!tails) return cudaErrorInvalidValue;
     CUtensorMap* maps = static_cast<CUtensorMap*>(d.scratch);
-    int32_t* split_offs = d.offsets ? nullptr : reinterpret_cast<int32_t*>(maps + 2 * d.num_groups);
-    {
+    p.split_rows = d.offsets ? 0 : d.split_rows;
+    // splits of a dense product start on k-block boundaries, so they need
+    // tail maps only when the whole range ends inside a k-block
+    if (d.offsets || d.split_rows % tc::BK != 0) {
       KernelScope ks("group_maps", c.stream);
       tc::build_group_maps<<<(d.num_groups + tc::kMapWarps - 1) / tc::kMapWarps, 32 * tc::kMapWarps, 0, c.stream>>>(
-          *tails, d.offsets, d.num_groups, d.split_rows, split_offs, static_cast<const uint8_t*>(d.A), pl.lda * 2,
+          *tails, d.offsets, d.num_groups, d.split_rows, static_cast<const uint8_t*>(d.A), pl.lda * 2,
           gb ? nullptr : static_cast<const uint8_t*>(d.B), pl.ldb * 2, maps);
+      cudaError_t st = cudaGetLastError();
+      if (st != cudaSuccess) return st;
     }
-    cudaError_t st = cudaGetLastError();
-    if (st != cudaSuccess) return st;
     p.gmaps = maps;
-    if (split_offs) p.offsets = split_offs;
   }
   KernelScope ks(name, c.stream);
   if (ga) return launch_inst<256, false, false, 1, 3, bf16, 2, 1>(c, p, ub);

@@ -49,6 +49,10 @@ struct Params {
   void* aux;
   uint32_t* err;
   const CUtensorMap* gmaps;  // Group::K: per group {A, B} maps of its last rows (fewer than BK)
+  int64_t split_rows;        // Group::K with offsets == nullptr: split g is rows
+                             // [lo(g), lo(g + 1)), lo(g) = split_rows g / G rounded down to a
+                             // multiple of BK (lo(G) = split_rows): only the last split can
+                             // end inside a k-block
   const int32_t* gather;     // GATHER: source row of each gathered row (the permutation's token_of_row)
 };
 
@@ -450,6 +454,88 @@ __device__ __forceinline__ void decode_tile(const Params& p, int t, const int* s
   ti.nkb = (int)((ti.kend - ti.kbeg + BK - 1) / BK);
 }
 
+// The tiles one walker (a CTA, or a CTA pair) takes, in order.  Dense and
+// Group::M GEMMs: tiles cta0, cta0 + ncta, ...  Group::K GEMMs (per-expert
+// weight gradients) cost in proportion to the group's rows, and a group
+// without rows only writes zeros, which needs no MMA and no accumulator.
+// There the prologue partitions the groups, stably, into the non-empty ones
+// and the empty ones, and every walker takes:
+//   * the non-empty groups' tiles round-robin over the walkers (round r takes
+//     tiles r * ncta .. r * ncta + ncta - 1, walker p the p-th), or, when the
+//     groups' k-block counts differ by more than a factor of two, in snake
+//     order (walker p the (ncta - 1 - p)-th of an odd round), which evens out
+//     the k-blocks per walker;
+//   * the empty groups' tiles p, p + ncta, ..., interleaved with its
+//     non-empty ones in proportion to the k-blocks done so far, so that the
+//     epilogue writes the zero tiles while the MMA works on the next tiles
+//     instead of in a write-only phase at the end.
+// On the skewed workload (94 of 128 experts empty, the largest ones at 32768
+// rows) this took the GEMM-1 weight gradient from 1.68 to 1.43 ms; on
+// balanced workloads the snake order measured 3-4 % slower than round-robin.
+// Producer, MMA issuer and epilogue warps of both CTAs of a pair walk the
+// same sequence.
+struct Walker {
+  int t, total, ncta, p;           // Dense / Group::M
+  int r, zi, nz, nc, nce, per;     // Group::K: next round, zero tiles taken / owned, non-empty tiles and groups
+  bool snake;                      // Group::K: snake order
+  int64_t cum, tot;                // Group::K: k-blocks taken / owned
+};
+
+__device__ __forceinline__ int kblocks(const int* s_off, int g) { return (s_off[g + 1] - s_off[g] + BK - 1) / BK; }
+__device__ __forceinline__ int walk_index(int r, int p, int ncta, bool snake) {
+  return r * ncta + ((snake && (r & 1)) ? ncta - 1 - p : p);
+}
+
+template <int GROUP>
+__device__ __forceinline__ Walker make_walker(int cta0, int ncta, int total, int per, int nce, int nz,
+                                              int64_t tot, bool snake) {
+  Walker w;
+  w.t = cta0 - ncta;
+  w.total = total;
+  w.ncta = ncta;
+  w.p = cta0;
+  w.r = 0;
+  w.zi = 0;
+  w.nz = nz;
+  w.nce = nce;
+  w.per = per;
+  w.nc = nce * per;
+  w.snake = snake;
+  w.cum = 0;
+  w.tot = tot;
+  return w;
+}
+
+// The walker's next tile (the index decode_tile takes); false when done.
+// s_ord (Group::K): the non-empty groups by index, then the empty ones.
+template <int GROUP>
+__device__ __forceinline__ bool next_tile(Walker& w, const int* s_off, const int* s_ord, int& t) {
+  if (GROUP != 2 || (!w.snake && w.nce * w.per == w.total)) {
+    // Dense, Group::M, or Group::K without empty groups in round-robin order
+    // (the partition is then the identity): tiles cta0, cta0 + ncta, ...
+    w.t += w.ncta;
+    t = w.t;
+    return w.t < w.total;
+  }
+  bool zero = w.zi < w.nz && (int64_t)w.zi * w.tot <= w.cum * w.nz;
+  if (!zero) {
+    const int c = walk_index(w.r, w.p, w.ncta, w.snake);
+    if (c < w.nc) {
+      const int g = s_ord[c / w.per];
+      t = g * w.per + c % w.per;
+      w.cum += kblocks(s_off, g);
+      ++w.r;
+      return true;
+    }
+    zero = w.zi < w.nz;
+  }
+  if (!zero) return false;
+  const int z = w.p + w.zi * w.ncta;
+  t = s_ord[w.nce + z / w.per] * w.per + z % w.per;
+  ++w.zi;
+  return true;
+}
+
 __device__ __forceinline__ int64_t imin64(int64_t a, int64_t b) { return a < b ? a : b; }
 __device__ __forceinline__ int64_t imax64(int64_t a, int64_t b) { return a > b ? a : b; }
 
@@ -511,6 +597,9 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
   __shared__ int s_pref[kMaxE + 1];
   __shared__ int s_total;
   __shared__ volatile int s_abort;
+  __shared__ int s_knce, s_knz;      // Group::K: non-empty groups; this walker's zero tiles
+  __shared__ int s_ksnake;           // Group::K: snake order
+  __shared__ long long s_ktot;       // Group::K: this walker's k-blocks
 
   const int tid = threadIdx.x;
   const int warp = tid >> 5, lane = tid & 31;
@@ -538,9 +627,66 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
     tmem_relinquish_cg<CG>();
   }
   if (GROUP != 0) {
-    for (int i = tid; i <= p.num_groups; i += C::kThreads) s_off[i] = p.offsets[i];
+    if (p.offsets) {
+      for (int i = tid; i <= p.num_groups; i += C::kThreads) s_off[i] = p.offsets[i];
+    } else {
+      for (int i = tid; i <= p.num_groups; i += C::kThreads)
+        s_off[i] = i < p.num_groups ? (int)((p.split_rows * i / p.num_groups) & ~(int64_t)(BK - 1))
+                                    : (int)p.split_rows;
+    }
   }
   __syncthreads();
+  if (GROUP == 2 && warp == 0) {
+    // s_pref: the non-empty groups by index, then the empty ones (a stable
+    // partition); the walker's share of the non-empty tiles' k-blocks and of
+    // the empty tiles; snake order when the k-block counts spread widely
+    const int G = p.num_groups;
+    const int per = p.tiles_m * p.tiles_n;
+    int nce = 0, kmin = 0x7fffffff, kmax = 0;
+    for (int j = lane; j < G; j += 32) {
+      const int kj = kblocks(s_off, j);
+      if (kj > 0) {
+        ++nce;
+        kmin = min(kmin, kj);
+        kmax = max(kmax, kj);
+      }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      nce += __shfl_xor_sync(0xffffffffu, nce, o);
+      kmin = min(kmin, __shfl_xor_sync(0xffffffffu, kmin, o));
+      kmax = max(kmax, __shfl_xor_sync(0xffffffffu, kmax, o));
+    }
+    int before_ne = 0, before_e = 0;
+    for (int j0 = 0; j0 < G; j0 += 32) {
+      const int j = j0 + lane;
+      const bool ne = j < G && kblocks(s_off, j) > 0;
+      const unsigned bne = __ballot_sync(0xffffffffu, ne), be = __ballot_sync(0xffffffffu, j < G && !ne);
+      const unsigned below = (1u << lane) - 1u;
+      if (j < G) s_pref[ne ? before_ne + __popc(bne & below) : nce + before_e + __popc(be & below)] = j;
+      before_ne += __popc(bne);
+      before_e += __popc(be);
+    }
+    __syncwarp();
+    const bool snake = nce > 0 && kmax > 2 * kmin;
+    const int nc = nce * per, nzt = (G - nce) * per;
+    long long tot = 0;
+    if (nzt > 0) {  // the walker's k-blocks pace its zero tiles
+      for (int r = lane;; r += 32) {
+        const int c = walk_index(r, cta0, ncta, snake);
+        if (c >= nc) break;
+        tot += kblocks(s_off, s_pref[c / per]);
+      }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) tot += __shfl_xor_sync(0xffffffffu, tot, o);
+    }
+    if (lane == 0) {
+      s_knce = nce;
+      s_ktot = tot;
+      s_knz = cta0 < nzt ? (nzt - cta0 + ncta - 1) / ncta : 0;
+      s_ksnake = snake ? 1 : 0;
+    }
+  }
   if (tid == 0) {
     if (GROUP == 0) {
       s_total = p.tiles_m * p.tiles_n;
@@ -562,6 +708,10 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
   tc_fence_after();
   const uint32_t tmem_base = *s_tmem;
   const int total = s_total;
+  const int kper = p.tiles_m * p.tiles_n;
+  const int knce = GROUP == 2 ? s_knce : 0, knz = GROUP == 2 ? s_knz : 0;
+  const int64_t ktot = GROUP == 2 ? (int64_t)s_ktot : 0;
+  const bool ksnake = GROUP == 2 && s_ksnake != 0;
 
   if (warp == 0 && GATHER != 0) {
     // ------------------------------------------------------------ producer (gathering, warp-wide)
@@ -570,7 +720,8 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
     int issued = 0;
     uint32_t last_phase = 0;
     bool ok = true;
-    for (int t = cta0; t < total && ok; t += ncta) {
+    Walker wk = make_walker<GROUP>(cta0, ncta, total, kper, knce, knz, ktot, ksnake);
+    for (int t; ok && next_tile<GROUP>(wk, s_off, s_pref, t);) {
       Tile ti;
       decode_tile<GROUP, CG>(p, t, s_off, s_pref, rank, ti);
       const int64_t nb = ti.n0 * BN + (int64_t)rank * BNC;
@@ -675,7 +826,8 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
       int issued = 0;
       uint32_t last_phase = 0;  // bit s: phase of the last copy issued into stage s
       bool ok = true;
-      for (int t = cta0; t < total && ok; t += ncta) {
+      Walker wk = make_walker<GROUP>(cta0, ncta, total, kper, knce, knz, ktot, ksnake);
+      for (int t; ok && next_tile<GROUP>(wk, s_off, s_pref, t);) {
         Tile ti;
         decode_tile<GROUP, CG>(p, t, s_off, s_pref, rank, ti);
         const int64_t nb = ti.n0 * BN + (int64_t)rank * BNC;  // this CTA's first B row / column
@@ -760,7 +912,8 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
     bool ok = true;
     bool issued_any = false;
     constexpr uint16_t kBoth = 0x3;
-    for (int t = cta0; t < total && ok && leader; t += ncta) {
+    Walker wk = make_walker<GROUP>(cta0, ncta, total, kper, knce, knz, ktot, ksnake);
+    for (int t; ok && leader && next_tile<GROUP>(wk, s_off, s_pref, t);) {
       Tile ti;
       decode_tile<GROUP, CG>(p, t, s_off, s_pref, rank, ti);
       if (ti.nkb == 0) continue;
@@ -812,7 +965,8 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
     const int64_t ldc_b = p.ldc * (int64_t)sizeof(TC);
     int acc = 0;
     uint32_t acc_phase = 0;
-    for (int t = cta0; t < total; t += ncta) {
+    Walker wk = make_walker<GROUP>(cta0, ncta, total, kper, knce, knz, ktot, ksnake);
+    for (int t; next_tile<GROUP>(wk, s_off, s_pref, t);) {
       Tile ti;
       decode_tile<GROUP, CG>(p, t, s_off, s_pref, rank, ti);
       const int64_t n0 = ti.n0 * BN;
@@ -1029,8 +1183,8 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
 // group's end, so the next group's rows never enter the reduction, and every
 // map's base lies inside its tensor.  out[2g] = A, out[2g + 1] = B (none for
 // a group whose row count is a multiple of BK).  With offsets == nullptr the
-// groups are G equal splits of [0, split_rows) and their offsets are written
-// to offs_out for the GEMM to read.
+// groups are the G splits of [0, split_rows) that the GEMM forms itself
+// (Params::split_rows), of which only the last can have a tail.
 // One warp per group: the template is copied into shared memory, its address
 // is replaced there (tensormap.replace on shared::cta), and the warp copies
 // the finished map to global memory with tensormap.cp_fenceproxy, which
@@ -1043,8 +1197,7 @@ struct TailTemplates {
 constexpr int kMapWarps = 4;
 __global__ void __launch_bounds__(32 * kMapWarps) build_group_maps(
     const __grid_constant__ TailTemplates tt, const int32_t* __restrict__ offsets, int G, int64_t split_rows,
-    int32_t* __restrict__ offs_out, const uint8_t* a_base, int64_t a_row_bytes, const uint8_t* b_base,
-    int64_t b_row_bytes, CUtensorMap* out) {
+    const uint8_t* a_base, int64_t a_row_bytes, const uint8_t* b_base, int64_t b_row_bytes, CUtensorMap* out) {
   __shared__ alignas(128) CUtensorMap sm[kMapWarps][2];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int g = blockIdx.x * kMapWarps + warp;
@@ -1054,12 +1207,8 @@ __global__ void __launch_bounds__(32 * kMapWarps) build_group_maps(
     lo = offsets[g];
     hi = offsets[g + 1];
   } else {
-    lo = split_rows * g / G;
-    hi = split_rows * (g + 1) / G;
-    if (lane == 0) {
-      offs_out[g] = (int32_t)lo;
-      if (g == G - 1) offs_out[G] = (int32_t)hi;
-    }
+    lo = (split_rows * g / G) & ~(int64_t)(BK - 1);
+    hi = g + 1 < G ? (split_rows * (g + 1) / G) & ~(int64_t)(BK - 1) : split_rows;
   }
   const int r = (int)((hi - lo) % BK);
   if (r == 0) return;  // no tail: every k-block of the group is whole

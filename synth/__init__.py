@@ -87,9 +87,14 @@ SKEW = Workload("skew_T32768_D2048_E128_K8_F1024", S=8192, GBS=4, D=2048, E=128,
 # ~768 rows per expert): a case for detailed profiler captures, which replay
 # each kernel many times and save and restore device memory around them.
 BASE_HALF = Workload("base_half_T4096_D2048_E32_K6_F1024", S=2048, GBS=2, D=2048, E=32, K=6, F=1024)
+# The skewed workload with half the tokens and half the experts (the same
+# logit-bias formula, so a similar head of near-capped experts and a tail of
+# empty ones): about 4 GB on the device, for detailed profiler captures.
+SKEW_HALF = Workload("skew_half_T16384_D2048_E64_K8_F1024", S=4096, GBS=4, D=2048, E=64, K=8, F=1024,
+                     skew_bias=True)
 
-WORKLOADS = {w.name: w for w in (TINY, BASE, CEMOE, LATENT, SKEW, BASE_HALF)}
-ALIASES = {"C1": TINY, "C2": BASE, "C3": CEMOE, "C4": LATENT, "C5": SKEW, "C2h": BASE_HALF}
+WORKLOADS = {w.name: w for w in (TINY, BASE, CEMOE, LATENT, SKEW, BASE_HALF, SKEW_HALF)}
+ALIASES = {"C1": TINY, "C2": BASE, "C3": CEMOE, "C4": LATENT, "C5": SKEW, "C2h": BASE_HALF, "C5h": SKEW_HALF}
 
 
 def get(name: str) -> Workload:
