@@ -93,8 +93,14 @@ BASE_HALF = Workload("base_half_T4096_D2048_E32_K6_F1024", S=2048, GBS=2, D=2048
 SKEW_HALF = Workload("skew_half_T16384_D2048_E64_K8_F1024", S=4096, GBS=4, D=2048, E=64, K=8, F=1024,
                      skew_bias=True)
 
-WORKLOADS = {w.name: w for w in (TINY, BASE, CEMOE, LATENT, SKEW, BASE_HALF, SKEW_HALF)}
-ALIASES = {"C1": TINY, "C2": BASE, "C3": CEMOE, "C4": LATENT, "C5": SKEW, "C2h": BASE_HALF, "C5h": SKEW_HALF}
+# LatentMoE with half the tokens and half the experts (the same ~512 rows per
+# expert): about 2.5 GB on the device, for detailed profiler captures.
+LATENT_HALF = Workload("latent_half_T8192_H4096_D1024_E128_K8_F768", S=4096, GBS=2, D=1024, E=128, K=8, F=768,
+                       H=4096)
+
+WORKLOADS = {w.name: w for w in (TINY, BASE, CEMOE, LATENT, SKEW, BASE_HALF, SKEW_HALF, LATENT_HALF)}
+ALIASES = {"C1": TINY, "C2": BASE, "C3": CEMOE, "C4": LATENT, "C5": SKEW, "C2h": BASE_HALF, "C5h": SKEW_HALF,
+           "C4h": LATENT_HALF}
 
 
 def get(name: str) -> Workload:
