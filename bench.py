@@ -435,7 +435,8 @@ def top_roofline(kernels: dict, w: synth.Workload, peaks: dict) -> dict:
 
 
 def measure(w: synth.Workload, args, rank: int, world: int, barrier, clocks=None, e2e_steps: int = 0,
-            steps: int | None = None, router: str = "softmax", shared_width: int = 0, payload: str = "bf16"):
+            steps: int | None = None, router: str = "softmax", shared_width: int = 0, payload: str = "bf16",
+            gather: bool = False):
     """Build one layer of workload ``w`` (this rank's seeded tokens), warm it
     up, capture its step as a CUDA graph and time ``steps`` steps twice: once
     with only per-step events (the headline), once with events around every
@@ -453,7 +454,7 @@ def measure(w: synth.Workload, args, rank: int, world: int, barrier, clocks=None
     if shared_width:
         inputs.update(synth.make_shared_expert(w, shared_width, rank_seed(w, rank)))
     L = MoeLayer(w.S, w.GBS, w.K, w.D, w.E, w.F, w.dtype, w.H, router=router, shared_F=shared_width,
-                 payload=payload)
+                 payload=payload, gather=gather)
     L.load(inputs)
     stream = torch.cuda.current_stream()
     flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device="cuda")
@@ -578,6 +579,9 @@ def main() -> None:
                          "NVFP4 (E2M1 codes, an E4M3 scale per 16 elements, a power-of-two scale per row)")
     ap.add_argument("--shared-width", type=int, default=0,
                     help="hidden units of the ungated shared expert (0 = none; Sec. 5.2)")
+    ap.add_argument("--gather", action="store_true",
+                    help="GEMM-1 and its weight gradient read the dispatched rows from x by token_of_row "
+                         "(no x_perm copy)")
     ap.add_argument("--router", default="softmax", choices=["softmax", "sigmoid"],
                     help="softmax top-K, or sigmoid scores + expert bias + sequence-level balance loss (Sec. 5.2)")
     args = ap.parse_args()
@@ -610,7 +614,7 @@ def main() -> None:
     peaks = _peaks()
     clocks = ClockSampler(local)
     r = measure(w, args, rank, world, barrier, clocks=clocks, e2e_steps=args.e2e_steps, router=args.router,
-                shared_width=args.shared_width, payload=args.payload)
+                shared_width=args.shared_width, payload=args.payload, gather=args.gather)
     clk = clocks.stop()
     T = r["T"]
     kernels = kernel_table(r["prof"], args.steps, w, T, args.shared_width, r["latent_fused"], peaks)
@@ -651,7 +655,7 @@ def main() -> None:
             "scaling": "weak", "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
             "config": {"workload": w.name, "T": T, "S": w.S, "GBS": w.GBS, "D": w.D, "E": w.E, "K": w.K, "F": w.F,
                        "H": w.H, "seed": w.seed, "router": args.router, "shared_width": args.shared_width,
-                       "payload": args.payload,
+                       "payload": args.payload, "gather": args.gather,
                        "parallelism": f"replicas x{world}, each rank its own tokens",
                        "launch": "one CUDA graph per step" if r["graph"] else "eager launches",
                        "l2": "256 MiB buffer written before every timed step (outside the step events); "

@@ -258,6 +258,15 @@ cudaError_t launch_gemm_tc(const Ctx& c, const GemmDesc& d, const char* name) {
   p.aux = d.aux;
   p.err = c.err;
   p.gather = d.gather;
+  if (ga) {
+    p.gsrc = static_cast<const uint8_t*>(d.A);
+    p.gsrc_ld = pl.lda * 2;
+    p.gsrc_rows = d.gather_rows;
+  } else if (gb) {
+    p.gsrc = static_cast<const uint8_t*>(d.B);
+    p.gsrc_ld = pl.ldb * 2;
+    p.gsrc_rows = d.gather_rows;
+  }
   int64_t ub;
   if (d.group == Group::Dense) ub = (int64_t)p.tiles_m * p.tiles_n;
   else if (d.group == Group::M) ub = ((d.max_rows + bmp - 1) / bmp + d.num_groups) * p.tiles_n;

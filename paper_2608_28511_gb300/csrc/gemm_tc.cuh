@@ -54,6 +54,9 @@ struct Params {
                              // multiple of BK (lo(G) = split_rows): only the last split can
                              // end inside a k-block
   const int32_t* gather;     // GATHER: source row of each gathered row (the permutation's token_of_row)
+  const uint8_t* gsrc;       // GATHER: the source matrix (bf16, row-major), its row pitch in bytes
+  int64_t gsrc_ld;           //   and its row count (source rows are checked against it)
+  int64_t gsrc_rows;
 };
 
 // ---------------------------------------------------------------------------
@@ -78,8 +81,11 @@ __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
 // pure write-after-read hand-off of TMEM: an epilogue thread arrives only after
 // tcgen05.wait::ld has returned its loads into registers and
 // tcgen05.fence::before_thread_sync has ordered them before the arrive, so the
-// MMA that then overwrites the accumulator cannot change what was read.  No
-// generic-proxy data is published through these barriers.
+// MMA that then overwrites the accumulator cannot change what was read.  The
+// one exception is the gathering producer, whose row copies are ordinary
+// (generic-proxy) writes: the other CTA of a pair forwards them with a proxy
+// fence and a cluster-scope release, and the MMA issuer waits on those full
+// barriers with mbar_try_wait_cluster and fences again before its MMAs.
 __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
   uint32_t ok;
   asm volatile(
@@ -91,18 +97,34 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
+// The same wait with acquire at cluster scope: for barriers on which the other
+// CTA of a pair publishes data written through the generic proxy (the row
+// copies of the gathering producer).
+__device__ __forceinline__ bool mbar_try_wait_cluster(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}\n"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
 __device__ __forceinline__ uint64_t global_timer_ns() {
   uint64_t t;
   asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
   return t;
 }
-// Wait for phase `parity` of `bar`; false if the CTA aborted or the limit expired.
+// Wait for phase `parity` of `bar`; false if the CTA aborted or the limit
+// expired.  cluster: acquire at cluster scope (mbar_try_wait_cluster).
 __device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, volatile int* abort_flag,
-                                             uint32_t* err) {
-  if (mbar_try_wait(bar, parity)) return true;
+                                             uint32_t* err, bool cluster = false) {
+  auto try_wait = [&]() { return cluster ? mbar_try_wait_cluster(bar, parity) : mbar_try_wait(bar, parity); };
+  if (try_wait()) return true;
   const uint64_t t0 = global_timer_ns();
   for (uint32_t i = 1;; ++i) {
-    if (mbar_try_wait(bar, parity)) return true;
+    if (try_wait()) return true;
     if ((i & 63u) == 0) {
       if (*abort_flag) return false;
       if (global_timer_ns() - t0 > kWaitLimitNs) {
@@ -214,6 +236,24 @@ __device__ __forceinline__ void tma_gather4_pair(uint32_t dst, const CUtensorMap
       "[%1, {%3, %4, %5, %6, %7}], [%2];" ::"r"(dst),
       "l"(reinterpret_cast<uint64_t>(map)), "r"(bar_cluster), "r"(x), "r"(r0), "r"(r1), "r"(r2), "r"(r3)
       : "memory");
+}
+// ---- row gathers by the producer warp's lanes (cp.async, 16 bytes each)
+// 16 bytes from global memory into shared memory, through L2 only; with
+// nbytes = 0 nothing is read and the 16 bytes are zero-filled.
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, uint32_t nbytes) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(nbytes) : "memory");
+}
+// An arrival on `bar` (this CTA) once all of this thread's earlier cp.async
+// copies have landed; the arrival counts toward the barrier's expected count.
+__device__ __forceinline__ void cp_async_arrive(uint32_t bar) {
+  asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;" ::: "memory"); }
+
+// Arrival on an mbarrier of either CTA of the cluster, releasing this
+// thread's earlier writes at cluster scope.
+__device__ __forceinline__ void mbar_arrive_release_cluster(uint32_t cluster_addr) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
 }
 template <int CG>
 __device__ __forceinline__ void tmem_alloc_cg(uint32_t dst_smem, uint32_t ncols) {
@@ -609,7 +649,12 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
 
   if (warp == 0 && lane == 0) {
     for (int s = 0; s < C::kStages; ++s) {
-      mbar_init(smem_u32(&full[s]), 1);
+      // gathering: the leader's expect_tx arrival, one arrival per producer
+      // lane of this CTA once its row copies into the stage have landed, and
+      // in a pair the other CTA's forwarded arrival; the other CTA of a pair
+      // counts only its own lanes' arrivals on its full barriers
+      const uint32_t cnt = GATHER == 0 ? 1u : CG == 1 ? 33u : (leader ? 34u : 32u);
+      mbar_init(smem_u32(&full[s]), cnt);
       mbar_init(smem_u32(&empty[s]), 1);
     }
     for (int a = 0; a < 2; ++a) {
@@ -715,33 +760,52 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
 
   if (warp == 0 && GATHER != 0) {
     // ------------------------------------------------------------ producer (gathering, warp-wide)
+    // The gathered operand's rows come from p.gsrc through p.gather, as 16-byte
+    // cp.async copies by the 32 lanes into the stage's 128-byte-swizzled
+    // layout (chunk c of row r at r * 128 + ((c ^ (r & 7)) << 4), the layout a
+    // tiled 128-byte-swizzle copy writes); lane 0 issues the other operand's
+    // tiled copies, which complete on the leader's full barrier as usual.
+    // Every lane then arrives on its CTA's full barrier of the stage once its
+    // copies have landed (cp.async.mbarrier.arrive), so the producer never
+    // waits for its own copies; in a pair the other CTA's MMA warp forwards
+    // its completed stages to the leader.
     int stage = 0;
     uint32_t phase = 0;
     int issued = 0;
     uint32_t last_phase = 0;
     bool ok = true;
+    const int q = lane >> 3, c = lane & 7;  // a warp instruction covers 4 rows of 8 chunks
+    auto src_row = [&](int64_t r) -> const uint8_t* {
+      int64_t src = r >= 0 ? (int64_t)__ldg(p.gather + r) : 0;
+      if (src < 0 || src >= p.gsrc_rows) {  // a bad row index: recorded, row 0 read instead
+        set_error(p.err, kErrIndex);
+        src = 0;
+      }
+      return p.gsrc + src * p.gsrc_ld;
+    };
     Walker wk = make_walker<GROUP>(cta0, ncta, total, kper, knce, knz, ktot, ksnake);
     for (int t; ok && next_tile<GROUP>(wk, s_off, s_pref, t);) {
       Tile ti;
       decode_tile<GROUP, CG>(p, t, s_off, s_pref, rank, ti);
       const int64_t nb = ti.n0 * BN + (int64_t)rank * BNC;
-      int ra[4] = {0, 0, 0, 0};  // GATHER 1: source rows of this tile's rows 4 lane .. 4 lane + 3
+      // GATHER 1: source rows of this CTA's A rows lane, lane + 32, lane + 64,
+      // lane + 96 (rows past the expert's end read row 0; their outputs are dropped)
+      const uint8_t* ra[4];
       if (GATHER == 1) {
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
-          const int64_t r = ti.row0 + 4 * lane + i;
-          ra[i] = r < ti.row_end ? __ldg(p.gather + r) : 0;  // rows past the expert's end are dropped later
+          const int64_t r = ti.row0 + lane + 32 * i;
+          ra[i] = src_row(r < ti.row_end ? r : -1);
         }
       }
       for (int kb = 0; kb < ti.nkb; ++kb) {
-        int okw = 1;
-        if (lane == 0) okw = wait_bounded(smem_u32(&empty[stage]), phase ^ 1u, &s_abort, p.err) ? 1 : 0;
-        okw = __shfl_sync(0xffffffffu, okw, 0);
-        if (!okw) { ok = false; break; }
+        // every lane observes the stage's release before its copies overwrite it
+        const bool okw = wait_bounded(smem_u32(&empty[stage]), phase ^ 1u, &s_abort, p.err);
+        if (!__all_sync(0xffffffffu, okw)) { ok = false; break; }
         const uint32_t fb_local = smem_u32(&full[stage]);
         const uint32_t fb = CG == 2 ? map_to_rank(fb_local, 0) : fb_local;
-        if (leader && lane == 0) mbar_expect_tx(fb_local, CG * C::kStageBytes);
-        __syncwarp();
+        // the leader expects the tiled operand's bytes of both CTAs
+        if (leader && lane == 0) mbar_expect_tx(fb_local, CG * (GATHER == 1 ? C::kBBytes : C::kABytes));
         const uint32_t sa = smem_u32(smem + stage * C::kStageBytes);
         const uint32_t sb = sa + C::kABytes;
         const int k0 = (int)(ti.kbeg + (int64_t)kb * BK);
@@ -749,13 +813,7 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
           if (CG == 2) tma_load_2d_pair(dst, m, fb, x, y);
           else tma_load_2d(dst, m, fb, x, y);
         };
-        auto gather4 = [&](uint32_t dst, const CUtensorMap* m, int x, const int* r) {
-          if (CG == 2) tma_gather4_pair(dst, m, fb, x, r[0], r[1], r[2], r[3]);
-          else tma_gather4(dst, m, fb, x, r[0], r[1], r[2], r[3]);
-        };
         if (GATHER == 1) {
-          // A: the tile's 128 rows from the source, 4 per lane
-          gather4(sa + lane * 512, &p.ta, k0, ra);
           if (lane == 0) {
             if (B_MN) {
               const int ky = (int)(ti.g * p.b_group_rows) + k0;
@@ -765,10 +823,17 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
               load(sb, &p.tb, k0, (int)(ti.g * p.b_group_rows + nb));
             }
           }
+          // A: 128 rows x 64 k (128 bytes) of the source rows, K-major
+#pragma unroll
+          for (int it = 0; it < BM / 4; ++it) {
+            const int r = 4 * it + q;
+            const uint8_t* base = reinterpret_cast<const uint8_t*>(
+                __shfl_sync(0xffffffffu, reinterpret_cast<uintptr_t>(ra[it >> 3]), r & 31));
+            cp_async16(sa + r * 128 + ((c ^ (r & 7)) << 4), base + (int64_t)k0 * 2 + c * 16, 16u);
+          }
         } else {
           // A: whole k-blocks from the full map, the group's last rows from
-          // its tail map (zero past the group's rows); B's 64 k rows from the
-          // source, in 64-column chunks of 16 four-row copies
+          // its tail map (zero past the group's rows)
           if (lane == 0) {
             if (kb < (int)((ti.kend - ti.kbeg) / BK)) {
               load(sa, &p.ta, (int)ti.row0, k0);
@@ -780,24 +845,33 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
               load(sa + 8192, ma, (int)ti.row0 + 64, 0);
             }
           }
+          // B: the block's 64 k rows (source rows through p.gather) x this
+          // CTA's BNC columns, MN-major in 64-column boxes of 8 KB; past the
+          // group's rows A is zero, so any valid source row will do; columns
+          // past N are zero-filled
+          const uint8_t* rb[2];
 #pragma unroll
-          for (int u = lane; u < (BNC / 64) * 16; u += 32) {
-            const int j = u >> 4, qd = u & 15;
-            int rb[4];
+          for (int i = 0; i < 2; ++i) {
+            const int64_t kr = (int64_t)k0 + lane + 32 * i;
+            rb[i] = src_row(kr < ti.kend ? kr : -1);
+          }
 #pragma unroll
-            for (int i = 0; i < 4; ++i) {
-              const int64_t kr = (int64_t)k0 + 4 * qd + i;
-              // past the group's rows A is zero, so any valid source row will do
-              rb[i] = kr < ti.kend ? __ldg(p.gather + kr) : 0;
-            }
-            gather4(sb + j * 8192 + qd * 512, &p.tb, (int)nb + 64 * j, rb);
+          for (int it = 0; it < (BNC / 64) * 16; ++it) {
+            const int j = it >> 4, r = (4 * it + q) & 63;
+            const uint8_t* base = reinterpret_cast<const uint8_t*>(
+                __shfl_sync(0xffffffffu, reinterpret_cast<uintptr_t>(rb[(it >> 3) & 1]), r & 31));
+            const int64_t col = nb + 64 * j + 8 * c;
+            const bool in = col < p.N;
+            cp_async16(sb + j * 8192 + r * 128 + ((c ^ (r & 7)) << 4), in ? base + col * 2 : p.gsrc, in ? 16u : 0u);
           }
         }
+        cp_async_arrive(fb_local);
         last_phase = (last_phase & ~(1u << stage)) | (phase << stage);
         ++issued;
         if (++stage == C::kStages) { stage = 0; phase ^= 1u; }
       }
     }
+    cp_async_wait_all();  // every copy lands before the CTA goes on
     // tail: wait until the MMA warp has released every stage this CTA filled.
     // Its releases are asynchronous arrivals (multicast to both CTAs of a pair)
     // that may still be in flight when the MMAs are done; waiting here keeps
@@ -922,7 +996,11 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
       tc_fence_after();
       const uint32_t d_tmem = tmem_base + (uint32_t)(acc * BN);
       for (int kb = 0; kb < ti.nkb; ++kb) {
-        if (!wait_bounded(smem_u32(&full[stage]), phase, &s_abort, p.err)) { ok = false; break; }
+        if (!wait_bounded(smem_u32(&full[stage]), phase, &s_abort, p.err, GATHER != 0 && CG == 2)) {
+          ok = false;
+          break;
+        }
+        if (GATHER != 0) fence_proxy_async_smem();  // the row copies, before the tensor core reads them
         tc_fence_after();
         const uint32_t sa = smem_u32(smem + stage * C::kStageBytes);
         const uint32_t sb = sa + C::kABytes;
@@ -945,6 +1023,24 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
       if (lane == 0) mma_commit_cg<CG>(smem_u32(&tfull[acc]), kBoth);
       __syncwarp();
       if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
+    }
+    if (GATHER != 0 && CG == 2 && !leader && lane == 0) {
+      // the other CTA of a pair: forward each stage whose row copies have all
+      // landed here (this CTA's full barrier) to the leader's full barrier
+      int fs = 0;
+      uint32_t fph = 0;
+      Walker fw = make_walker<GROUP>(cta0, ncta, total, kper, knce, knz, ktot, ksnake);
+      bool fok = true;
+      for (int t; fok && next_tile<GROUP>(fw, s_off, s_pref, t);) {
+        Tile ti;
+        decode_tile<GROUP, CG>(p, t, s_off, s_pref, rank, ti);
+        for (int kb = 0; kb < ti.nkb; ++kb) {
+          if (!wait_bounded(smem_u32(&full[fs]), fph, &s_abort, p.err)) { fok = false; break; }
+          fence_proxy_async_smem();
+          mbar_arrive_release_cluster(map_to_rank(smem_u32(&full[fs]), 0));
+          if (++fs == C::kStages) { fs = 0; fph ^= 1u; }
+        }
+      }
     }
     // drain: all MMAs issued by this warp have completed before TMEM is freed
     if (lane == 0 && issued_any) {
