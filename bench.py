@@ -570,7 +570,7 @@ def main() -> None:
     ap.add_argument("--ref-tokens", type=int, default=0, help="fixed oracle tokens per step (0 = sized to time)")
     ap.add_argument("--cpu-budget", type=float, default=15.0, help="seconds of CPU work for cpu_baseline")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--e2e-steps", type=int, default=30,
+    ap.add_argument("--e2e-steps", type=int, default=60,
                     help="timed end-to-end steps (their first upload and last download are not overlapped)")
     ap.add_argument("--no-graph", action="store_true",
                     help="launch every kernel from the host each step instead of replaying a captured CUDA graph")

@@ -1122,11 +1122,11 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
           const int64_t cb = n0 + blk * 128;
           if (cb >= p.N) break;
           {
-            float u[32], a[32];
+            // g (in v) and u are stored first; a = silu(g) * u then overwrites v,
+            // so only two 32-value rows are live at a time
+            float u[32];
             tmem_ld32(tbase + blk * 128 + half * 32, v);
             tmem_ld32(tbase + blk * 128 + 64 + half * 32, u);
-#pragma unroll
-            for (int i = 0; i < 32; ++i) a[i] = silu_f(v[i]) * u[i];
 #pragma unroll
             for (int i = 0; i < NP; ++i) pk[i] = pack16<TC>(v + i * Vec<TC>::N);
             __syncwarp();
@@ -1140,7 +1140,9 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
             __syncwarp();
             stage_store<RB>(stg, lane, c_rows + (cb + 64 + half * 32) * sizeof(TC), ldc_b, nrows);
 #pragma unroll
-            for (int i = 0; i < NP; ++i) pk[i] = pack16<TC>(a + i * Vec<TC>::N);
+            for (int i = 0; i < 32; ++i) v[i] = silu_f(v[i]) * u[i];
+#pragma unroll
+            for (int i = 0; i < NP; ++i) pk[i] = pack16<TC>(v + i * Vec<TC>::N);
             __syncwarp();
             stage_put<RB>(stg, lane, pk);
             __syncwarp();
