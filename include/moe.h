@@ -200,10 +200,11 @@ int moe_expert_ffn(const moe_shape_t* shape, const void* x_perm, const int32_t* 
 
 /* moe_expert_ffn with GEMM-1 reading its rows straight from the dispatch
  * input: row r of expert e is x[token_of_row[r]] (x [T, D]; for LatentMoE the
- * down-projected x_lat), loaded by the copy engine's four-row gathers, so the
- * dispatched copy x_perm is never written (moe_dispatch may then be called
- * with x_perm = NULL).  Same results as moe_expert_ffn on
- * x_perm = x[token_of_row]. */
+ * down-projected x_lat), copied row by row by the GEMM's producer (16-byte
+ * cp.async copies), so the dispatched copy x_perm is never written
+ * (moe_dispatch may then be called with x_perm = NULL).  Same results as
+ * moe_expert_ffn on x_perm = x[token_of_row]; slower on GB300 than the tiled
+ * copies of x_perm. */
 int moe_expert_ffn_gather(const moe_shape_t* shape, const void* x, const int32_t* token_of_row,
                           const int32_t* expert_offsets, const void* w1, const void* w2, void* h_save,
                           void* act_save, void* y_perm, void* ws, size_t ws_bytes, void* stream);

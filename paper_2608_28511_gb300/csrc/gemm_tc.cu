@@ -227,8 +227,8 @@ cudaError_t launch_gemm_tc(const Ctx& c, const GemmDesc& d, const char* name) {
   memset(&p, 0, sizeof(p));
   const int bn = pl.bn, bmp = BM * pl.cg, bnc = bn / pl.cg;
   // A: K-major box {64 k, 128 m}; MN-major box {64 m, 64 k}
-  const bool ga = d.gather && d.group == Group::M;  // A's rows gathered (one-row box)
-  const bool gb = d.gather && d.group == Group::K;  // B's k rows gathered (one-row box)
+  const bool ga = d.gather && d.group == Group::M;  // A's rows gathered (cp.async row copies; its map unused)
+  const bool gb = d.gather && d.group == Group::K;  // B's k rows gathered (cp.async row copies; its map unused)
   int64_t a_rows = pl.a_mn ? (d.group == Group::K ? d.max_rows : d.K) : (d.group == Group::M ? d.max_rows : d.M);
   if (ga) a_rows = d.gather_rows;
   const int64_t a_inner = pl.a_mn ? d.M : d.K;
