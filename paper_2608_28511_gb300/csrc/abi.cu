@@ -172,9 +172,11 @@ size_t align_up(size_t v) { return (v + 255) & ~size_t(255); }
 // Workspace carve-up.  Calls are ordered on one stream, so the regions used by
 // different calls may overlap.
 size_t ws_perm(const Dims& d) { return align_up(perm_workspace_bytes(d.TK, d.E)); }
-// dH [TK, 2F], dA [TK, F], then the wgrad GEMMs' per-expert tail tensor maps
+// dH [TK, 2F], dA [TK, F], then the two wgrad GEMMs' per-expert tail tensor
+// maps (one region each: one launch builds both)
 size_t ws_ffn_bwd_maps_offset(const Dims& d) { return align_up((size_t)d.TK * 3 * d.F * d.bx); }
-size_t ws_ffn_bwd(const Dims& d) { return ws_ffn_bwd_maps_offset(d) + align_up(gemm_tc_group_scratch_bytes(d.E)); }
+size_t ws_ffn_bwd_maps_bytes(const Dims& d) { return align_up(gemm_tc_group_scratch_bytes(d.E)); }
+size_t ws_ffn_bwd(const Dims& d) { return ws_ffn_bwd_maps_offset(d) + 2 * ws_ffn_bwd_maps_bytes(d); }
 // Router weight gradient: split-K over the T tokens into at most kRouterSplits
 // fp32 partial products, summed in order afterwards.
 constexpr int kRouterSplits = 16;
@@ -594,6 +596,7 @@ static int expert_ffn_bwd_impl(const Ctx& c, const Dims& d, const void* dy_perm,
   void* dH = ws;
   void* dA = static_cast<char*>(ws) + (size_t)d.TK * 2 * d.F * d.bx;
   void* maps = static_cast<char*>(ws) + ws_ffn_bwd_maps_offset(d);
+  void* maps1 = static_cast<char*>(maps) + ws_ffn_bwd_maps_bytes(d);
   // dgrad-2: dA = dy_perm . w2_e, then the SwiGLU backward dA, h -> dH
   GemmDesc a;
   a.group = Group::M;
@@ -677,7 +680,7 @@ static int expert_ffn_bwd_impl(const Ctx& c, const Dims& d, const void* dy_perm,
   w.gather = gather;
   w.gather_rows = d.T;
   w.max_rows = d.TK;
-  w.scratch = maps;
+  w.scratch = maps1;
   w.C = dw1;
   w.c_type = DType::F32;
   w.ldc = d.D;
@@ -685,6 +688,13 @@ static int expert_ffn_bwd_impl(const Ctx& c, const Dims& d, const void* dy_perm,
   if (d.TK > 0) {
     TRY_CUDA(gemm(c, a, "ffn2_dgrad_tc", "ffn2_dgrad_simt"));
     TRY_CUDA(launch_swiglu_bwd(c, d.dt, dA, h_save, d.TK, d.F, dH));
+  }
+  // both weight gradients' tail maps in one launch (each GEMM builds its own
+  // if they are not both on the tensor-core engine)
+  cudaError_t maps_st = cudaSuccess;
+  if (gemm_tc_group_maps_pair(c, b, w, &maps_st)) {
+    TRY_CUDA(maps_st);
+    b.maps_ready = w.maps_ready = true;
   }
   TRY_CUDA(gemm(c, b, "ffn2_wgrad_tc", "ffn2_wgrad_simt"));
   TRY_CUDA(gemm(c, w, "ffn1_wgrad_tc", "ffn1_wgrad_simt"));

@@ -281,7 +281,7 @@ cudaError_t launch_gemm_tc(const Ctx& c, const GemmDesc& d, const char* name) {
     p.split_rows = d.offsets ? 0 : d.split_rows;
     // splits of a dense product start on k-block boundaries, so they need
     // tail maps only when the whole range ends inside a k-block
-    if (d.offsets || d.split_rows % tc::BK != 0) {
+    if (!d.maps_ready && (d.offsets || d.split_rows % tc::BK != 0)) {
       KernelScope ks("group_maps", c.stream);
       tc::build_group_maps<<<(d.num_groups + tc::kMapWarps - 1) / tc::kMapWarps, 32 * tc::kMapWarps, 0, c.stream>>>(
           *tails, d.offsets, d.num_groups, d.split_rows, static_cast<const uint8_t*>(d.A), pl.lda * 2,
@@ -321,6 +321,39 @@ cudaError_t launch_gemm_tc(const Ctx& c, const GemmDesc& d, const char* name) {
   if (g == 0 && !pl.a_mn && pl.b_mn && e == 2) return launch_inst<256, false, true, 0, 2, bf16, 1>(c, p, ub);
   if (g == 0 && pl.a_mn && pl.b_mn) return launch_inst<256, true, true, 0, 0, float, 1>(c, p, ub);
   return cudaErrorNotSupported;
+}
+
+bool gemm_tc_group_maps_pair(const Ctx& c, const GemmDesc& d0, const GemmDesc& d1, cudaError_t* err) {
+  *err = cudaSuccess;
+  const GemmDesc* ds[2] = {&d0, &d1};
+  Plan pl[2];
+  const tc::TailTemplates* tails[2];
+  for (int k = 0; k < 2; ++k) {
+    const GemmDesc& d = *ds[k];
+    if (d.group != Group::K || !d.offsets || !d.scratch || !make_plan(d, &pl[k]) || !gemm_tc_supports(d))
+      return false;
+    const bool gb = d.gather != nullptr;
+    tails[k] = tail_templates(d.A, pl[k].a_mn ? d.M : d.K, pl[k].lda * 2, gb ? nullptr : d.B,
+                              pl[k].b_mn ? d.N : d.K, pl[k].ldb * 2);
+    if (!tails[k]) return false;
+  }
+  if (d0.offsets != d1.offsets || d0.num_groups != d1.num_groups || d0.num_groups <= 0) return false;
+  static thread_local tc::TailTemplatesPair tt;  // 32 KB: not on the stack
+  for (int k = 0; k < 2; ++k) {
+    memcpy(tt.a[k], &tails[k]->a[1], sizeof(tt.a[k]));
+    memcpy(tt.b[k], &tails[k]->b[1], sizeof(tt.b[k]));
+  }
+  const int G = d0.num_groups;
+  auto bbase = [&](int k) {
+    return ds[k]->gather ? nullptr : static_cast<const uint8_t*>(ds[k]->B);
+  };
+  KernelScope ks("group_maps", c.stream);
+  tc::build_group_maps_pair<<<(2 * G + tc::kMapWarps - 1) / tc::kMapWarps, 32 * tc::kMapWarps, 0, c.stream>>>(
+      tt, d0.offsets, G, static_cast<const uint8_t*>(d0.A), pl[0].lda * 2, bbase(0), pl[0].ldb * 2,
+      static_cast<CUtensorMap*>(d0.scratch), static_cast<const uint8_t*>(d1.A), pl[1].lda * 2, bbase(1),
+      pl[1].ldb * 2, static_cast<CUtensorMap*>(d1.scratch));
+  *err = cudaGetLastError();
+  return true;
 }
 
 }  // namespace moe

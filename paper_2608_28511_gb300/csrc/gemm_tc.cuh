@@ -1274,7 +1274,56 @@ struct TailTemplates {
   CUtensorMap a[BK];  // [r]: r rows (r = 1 .. BK - 1)
   CUtensorMap b[BK];
 };
+// The tail templates of two Group::K GEMMs (index r - 1 for r rows), for one
+// launch that builds the maps of both: 4 x 63 maps fit the 32764-byte kernel
+// parameter limit with the launch's other arguments.
+struct TailTemplatesPair {
+  CUtensorMap a[2][BK - 1];
+  CUtensorMap b[2][BK - 1];
+};
+static_assert(sizeof(TailTemplatesPair) + 256 <= 32764, "kernel parameter limit");
 constexpr int kMapWarps = 4;
+
+// One group's tail maps, by one warp: the templates for its r = (hi - lo) % BK
+// rows (ta1[r - 1], tb1[r - 1]; tb1 unused without b_base) moved to the
+// group's first tail row and copied to out2[0], out2[1].
+__device__ __forceinline__ void build_tail_maps(CUtensorMap* sm, int lane, const CUtensorMap* ta1,
+                                                const CUtensorMap* tb1, int64_t lo, int64_t hi,
+                                                const uint8_t* a_base, int64_t a_row_bytes, const uint8_t* b_base,
+                                                int64_t b_row_bytes, CUtensorMap* out2) {
+  const int r = (int)((hi - lo) % BK);
+  if (r == 0) return;  // no tail: every k-block of the group is whole
+  const int64_t first = hi - r;
+  const bool has_b = b_base != nullptr;  // NULL: B is gathered row by row (no tail B map)
+  // 32 lanes x 4 bytes = one 128-byte map
+  reinterpret_cast<uint32_t*>(&sm[0])[lane] = reinterpret_cast<const uint32_t*>(&ta1[r - 1])[lane];
+  if (has_b) reinterpret_cast<uint32_t*>(&sm[1])[lane] = reinterpret_cast<const uint32_t*>(&tb1[r - 1])[lane];
+  __syncwarp();
+  const uint32_t sa = smem_u32(&sm[0]), sb = smem_u32(&sm[1]);
+  if (lane == 0) {
+    const uint64_t pa = reinterpret_cast<uint64_t>(a_base + first * a_row_bytes);
+    asm volatile("tensormap.replace.tile.global_address.shared::cta.b1024.b64 [%0], %1;" ::"r"(sa), "l"(pa)
+                 : "memory");
+    if (has_b) {
+      const uint64_t pb = reinterpret_cast<uint64_t>(b_base + first * b_row_bytes);
+      asm volatile("tensormap.replace.tile.global_address.shared::cta.b1024.b64 [%0], %1;" ::"r"(sb), "l"(pb)
+                   : "memory");
+    }
+  }
+  __syncwarp();
+  asm volatile(
+      "tensormap.cp_fenceproxy.global.shared::cta.tensormap::generic.release.gpu.sync.aligned [%0], [%1], 128;" ::"l"(
+          reinterpret_cast<uint64_t>(out2)),
+      "r"(sa)
+      : "memory");
+  if (has_b)
+    asm volatile(
+        "tensormap.cp_fenceproxy.global.shared::cta.tensormap::generic.release.gpu.sync.aligned [%0], [%1], 128;" ::
+            "l"(reinterpret_cast<uint64_t>(out2 + 1)),
+        "r"(sb)
+        : "memory");
+}
+
 __global__ void __launch_bounds__(32 * kMapWarps) build_group_maps(
     const __grid_constant__ TailTemplates tt, const int32_t* __restrict__ offsets, int G, int64_t split_rows,
     const uint8_t* a_base, int64_t a_row_bytes, const uint8_t* b_base, int64_t b_row_bytes, CUtensorMap* out) {
@@ -1290,37 +1339,29 @@ __global__ void __launch_bounds__(32 * kMapWarps) build_group_maps(
     lo = (split_rows * g / G) & ~(int64_t)(BK - 1);
     hi = g + 1 < G ? (split_rows * (g + 1) / G) & ~(int64_t)(BK - 1) : split_rows;
   }
-  const int r = (int)((hi - lo) % BK);
-  if (r == 0) return;  // no tail: every k-block of the group is whole
-  const int64_t first = hi - r;
-  const bool has_b = b_base != nullptr;  // NULL: B is gathered through one full map (no tail B map)
-  // 32 lanes x 4 bytes = one 128-byte map
-  reinterpret_cast<uint32_t*>(&sm[warp][0])[lane] = reinterpret_cast<const uint32_t*>(&tt.a[r])[lane];
-  if (has_b) reinterpret_cast<uint32_t*>(&sm[warp][1])[lane] = reinterpret_cast<const uint32_t*>(&tt.b[r])[lane];
-  __syncwarp();
-  const uint32_t sa = smem_u32(&sm[warp][0]), sb = smem_u32(&sm[warp][1]);
-  if (lane == 0) {
-    const uint64_t pa = reinterpret_cast<uint64_t>(a_base + first * a_row_bytes);
-    asm volatile("tensormap.replace.tile.global_address.shared::cta.b1024.b64 [%0], %1;" ::"r"(sa), "l"(pa)
-                 : "memory");
-    if (has_b) {
-      const uint64_t pb = reinterpret_cast<uint64_t>(b_base + first * b_row_bytes);
-      asm volatile("tensormap.replace.tile.global_address.shared::cta.b1024.b64 [%0], %1;" ::"r"(sb), "l"(pb)
-                   : "memory");
-    }
-  }
-  __syncwarp();
-  asm volatile(
-      "tensormap.cp_fenceproxy.global.shared::cta.tensormap::generic.release.gpu.sync.aligned [%0], [%1], 128;" ::"l"(
-          reinterpret_cast<uint64_t>(out + 2 * g)),
-      "r"(sa)
-      : "memory");
-  if (has_b)
-    asm volatile(
-        "tensormap.cp_fenceproxy.global.shared::cta.tensormap::generic.release.gpu.sync.aligned [%0], [%1], 128;" ::
-            "l"(reinterpret_cast<uint64_t>(out + 2 * g + 1)),
-        "r"(sb)
-        : "memory");
+  build_tail_maps(sm[warp], lane, &tt.a[1], &tt.b[1], lo, hi, a_base, a_row_bytes, b_base, b_row_bytes,
+                  out + 2 * g);
+}
+
+// The tail maps of two Group::K GEMMs over the same groups (the two expert
+// weight gradients), in one launch: warp w builds GEMM w / G's maps of group
+// w % G.
+__global__ void __launch_bounds__(32 * kMapWarps) build_group_maps_pair(
+    const __grid_constant__ TailTemplatesPair tt, const int32_t* __restrict__ offsets, int G,
+    const uint8_t* a_base0, int64_t a_row_bytes0, const uint8_t* b_base0, int64_t b_row_bytes0, CUtensorMap* out0,
+    const uint8_t* a_base1, int64_t a_row_bytes1, const uint8_t* b_base1, int64_t b_row_bytes1, CUtensorMap* out1) {
+  __shared__ alignas(128) CUtensorMap sm[kMapWarps][2];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int w = blockIdx.x * kMapWarps + warp;
+  if (w >= 2 * G) return;  // the whole warp
+  const int k = w / G, g = w - k * G;
+  const int64_t lo = offsets[g], hi = offsets[g + 1];
+  if (k == 0)
+    build_tail_maps(sm[warp], lane, tt.a[0], tt.b[0], lo, hi, a_base0, a_row_bytes0, b_base0, b_row_bytes0,
+                    out0 + 2 * g);
+  else
+    build_tail_maps(sm[warp], lane, tt.a[1], tt.b[1], lo, hi, a_base1, a_row_bytes1, b_base1, b_row_bytes1,
+                    out1 + 2 * g);
 }
 
 }  // namespace tc

@@ -157,6 +157,8 @@ struct GemmDesc {
   void* aux = nullptr;               // SwigluFwd / ReluSqFwd activation output (c_type)
   void* scratch = nullptr;           // Group::K on the tensor-core engine: per-group tensor maps
                                      // (gemm_tc_group_scratch_bytes, 128-byte aligned)
+  bool maps_ready = false;           // Group::K: the maps in scratch were already built
+                                     // (gemm_tc_group_maps_pair)
   int64_t split_rows = 0;            // Group::K with offsets == nullptr: num_groups equal splits of
                                      // [0, split_rows) (split-K of a dense product)
   const int32_t* gather = nullptr;   // row indirection into a source matrix of gather_rows rows:
@@ -171,5 +173,10 @@ cudaError_t launch_gemm_simt(const Ctx& c, const GemmDesc& d, const char* name);
 bool gemm_tc_supports(const GemmDesc& d);
 size_t gemm_tc_group_scratch_bytes(int num_groups);
 cudaError_t launch_gemm_tc(const Ctx& c, const GemmDesc& d, const char* name);
+// Builds the per-group tail maps of two Group::K GEMMs over the same groups
+// (the two expert weight gradients) in one launch, into d0.scratch and
+// d1.scratch.  Returns false, launching nothing, unless both are tensor-core
+// GEMMs grouped by expert offsets; *err receives the launch status.
+bool gemm_tc_group_maps_pair(const Ctx& c, const GemmDesc& d0, const GemmDesc& d1, cudaError_t* err);
 
 }  // namespace moe
