@@ -58,7 +58,7 @@ def kernel_work(name: str, w: synth.Workload, T: int, Fs: int = 0, latent_fused:
     base = name.rsplit("_", 1)[0] if name.endswith(("_tc", "_simt")) else name
     flops = {
         "ffn1_swiglu": 4.0 * TK * D * F, "ffn2": 2.0 * TK * F * D, "ffn2_dgrad": 2.0 * TK * D * F,
-        "ffn2_wgrad": 2.0 * TK * D * F, "ffn1_dgrad": 4.0 * TK * F * D, "ffn1_wgrad": 4.0 * TK * F * D,
+        "ffn2_dgrad_swiglu": 2.0 * TK * D * F, "ffn2_wgrad": 2.0 * TK * D * F, "ffn1_dgrad": 4.0 * TK * F * D, "ffn1_wgrad": 4.0 * TK * F * D,
         "latent_fwd": 2.0 * T * w.H * D, "latent_dgrad": 2.0 * T * w.H * (D + (E if latent_fused else 0)),
         "latent_wgrad": 2.0 * T * w.H * D,
         "router_dgrad": 2.0 * T * Din * E, "router_wgrad": 2.0 * T * Din * E,
@@ -105,6 +105,8 @@ def gemm_bytes(name: str, w: synth.Workload, T: int, Fs: int = 0, latent_fused: 
         "ffn1_swiglu": (TK * D + E * 2 * F * D + TK * 3 * F) * bx,
         "ffn2": (TK * F + E * D * F + TK * D) * bx,
         "ffn2_dgrad": (TK * D + E * D * F + TK * F) * bx,
+        # the SwiGLU backward in the epilogue: h read, dH written instead of dA
+        "ffn2_dgrad_swiglu": (TK * D + E * D * F + TK * 4 * F) * bx,
         "ffn2_wgrad": (TK * F + TK * D) * bx + E * D * F * 4,
         "ffn1_dgrad": (TK * 2 * F + E * 2 * F * D + TK * D) * bx,
         "ffn1_wgrad": (TK * 2 * F + TK * D) * bx + E * 2 * F * D * 4,

@@ -686,8 +686,19 @@ static int expert_ffn_bwd_impl(const Ctx& c, const Dims& d, const void* dy_perm,
   w.ldc = d.D;
   w.sc_g = (int64_t)2 * d.F * d.D;
   if (d.TK > 0) {
-    TRY_CUDA(gemm(c, a, "ffn2_dgrad_tc", "ffn2_dgrad_simt"));
-    TRY_CUDA(launch_swiglu_bwd(c, d.dt, dA, h_save, d.TK, d.F, dH));
+    // on the tensor-core engine the SwiGLU backward runs in dgrad-2's epilogue
+    // (dA stays in TMEM: h in, dH out); otherwise as a separate pass over dA
+    GemmDesc af = a;
+    af.epi = Epi::SwigluBwd;
+    af.aux = const_cast<void*>(h_save);
+    af.C = dH;
+    af.ldc = 2 * d.F;
+    if (gemm_tc_supports(af)) {
+      TRY_CUDA(launch_gemm_tc(c, af, "ffn2_dgrad_swiglu_tc"));
+    } else {
+      TRY_CUDA(gemm(c, a, "ffn2_dgrad_tc", "ffn2_dgrad_simt"));
+      TRY_CUDA(launch_swiglu_bwd(c, d.dt, dA, h_save, d.TK, d.F, dH));
+    }
   }
   // both weight gradients' tail maps in one launch (each GEMM builds its own
   // if they are not both on the tensor-core engine)

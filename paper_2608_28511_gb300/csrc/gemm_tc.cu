@@ -117,6 +117,9 @@ bool make_plan(const GemmDesc& d, Plan* pl) {
     case Epi::ReluSqFwd:
       if (d.c_type != DType::BF16 || d.N % 64 || !d.aux || !al16(d.aux)) return false;
       break;
+    case Epi::SwigluBwd:
+      if (d.c_type != DType::BF16 || d.N % 64 || !d.aux || !al16(d.aux) || d.ldc != 2 * d.N) return false;
+      break;
   }
   pl->bn = 256;
   pl->cg = 1;
@@ -154,7 +157,7 @@ int max_pair_clusters(KernelT k, int smem, int threads) {
 template <int BN, bool A_MN, bool B_MN, int GROUP, int EPI, typename TC, int CG, int GATHER = 0>
 cudaError_t launch_inst(const Ctx& c, const Params& p, int64_t ub) {
   auto k = tc::gemm_tc_kernel<BN, A_MN, B_MN, GROUP, EPI, TC, CG, GATHER>;
-  constexpr int kSmem = Cfg<BN, CG, sizeof(TC)>::kSmem;
+  constexpr int kSmem = Cfg<BN, CG, sizeof(TC), EPI>::kSmem;
   constexpr int kThreads = Cfg<BN, CG, sizeof(TC)>::kThreads;
   static bool configured = false;
   static int pairs = 0;
@@ -212,6 +215,7 @@ bool gemm_tc_supports(const GemmDesc& d) {
   if (g == 1 && !pl.a_mn && !pl.b_mn && e == 3 && !f32) return true;
   if (g == 1 && !pl.a_mn && !pl.b_mn && e == 0 && !f32) return true;
   if (g == 1 && !pl.a_mn && pl.b_mn && e == 0 && !f32) return true;
+  if (g == 1 && !pl.a_mn && pl.b_mn && e == 5 && !f32) return true;
   if (g == 2 && pl.a_mn && pl.b_mn && e == 0 && f32) return true;
   if (g == 0 && !pl.a_mn && !pl.b_mn && e == 1 && f32) return true;
   if (g == 0 && !pl.a_mn && !pl.b_mn && (e == 0 || e == 2 || e == 4) && !f32) return true;
@@ -300,6 +304,7 @@ cudaError_t launch_gemm_tc(const Ctx& c, const GemmDesc& d, const char* name) {
     if (g == 1 && !pl.b_mn && e == 3) return launch_inst<256, false, false, 1, 3, bf16, 2>(c, p, ub);
     if (g == 1 && !pl.b_mn && e == 0) return launch_inst<256, false, false, 1, 0, bf16, 2>(c, p, ub);
     if (g == 1 && pl.b_mn && e == 0) return launch_inst<256, false, true, 1, 0, bf16, 2>(c, p, ub);
+    if (g == 1 && pl.b_mn && e == 5) return launch_inst<256, false, true, 1, 5, bf16, 2>(c, p, ub);
     if (g == 0 && !pl.a_mn && !pl.b_mn && e == 0) return launch_inst<256, false, false, 0, 0, bf16, 2>(c, p, ub);
     if (g == 0 && !pl.a_mn && !pl.b_mn && e == 2) return launch_inst<256, false, false, 0, 2, bf16, 2>(c, p, ub);
     if (g == 0 && !pl.a_mn && !pl.b_mn && e == 4) return launch_inst<256, false, false, 0, 4, bf16, 2>(c, p, ub);

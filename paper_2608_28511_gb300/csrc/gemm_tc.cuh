@@ -231,6 +231,38 @@ __device__ __forceinline__ void cp_async_arrive(uint32_t bar) {
   asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];" ::"r"(bar) : "memory");
 }
 __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait_group() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
+
+__device__ __forceinline__ uint4 lds128(uint32_t a) {
+  uint4 v;
+  asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(a) : "memory");
+  return v;
+}
+__device__ __forceinline__ void sts128(uint32_t a, const uint4& v) {
+  asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(a), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w) : "memory");
+}
+// EPI 5 slots: a 32-row x 32-byte block (16 bf16 columns) at byte
+// r * 32 + 16 (piece ^ (r / 4 mod 2)): conflict-free for a lane reading its own
+// row and for 4 rows x 2 pieces per quarter of a copy instruction.
+__device__ __forceinline__ uint32_t hs_off(int r, int pc) { return r * 32 + ((pc ^ ((r >> 2) & 1)) << 4); }
+// cp.async of the gate block (columns gcol .. gcol + 15) and the up block
+// (gcol + 64 ..) of rows 0 .. nrows - 1 into a slot (gate at +0, up at +1024);
+// one commit group.
+__device__ __forceinline__ void h_fetch(uint32_t slot, const uint8_t* rows, int64_t ld_b, int64_t gcol, int lane,
+                                        int nrows) {
+#pragma unroll
+  for (int it = 0; it < 2; ++it) {
+    const int r = it * 16 + lane / 2, pc = lane % 2;
+    if (r < nrows) {
+      const uint8_t* src = rows + r * ld_b + gcol * 2 + pc * 16;
+      cp_async16(slot + hs_off(r, pc), src, 16u);
+      cp_async16(slot + 1024 + hs_off(r, pc), src + 128, 16u);
+    }
+  }
+  cp_async_commit();
+}
 
 // Arrival on an mbarrier of either CTA of the cluster, releasing this
 // thread's earlier writes at cluster scope.
@@ -344,13 +376,14 @@ __host__ __device__ constexpr uint32_t make_idesc(int bn, int bm, bool a_mn, boo
 // CG = 1: one CTA computes a 128 x BN tile.  CG = 2: a cluster of two CTAs
 // computes a 256 x BN tile; each CTA stages its 128 rows of A and BN / 2 rows
 // of B, and holds its 128 accumulator rows in its own TMEM.
-template <int BN, int CG = 1, int TCB = 2>  // TCB: bytes per element of C
+template <int BN, int CG = 1, int TCB = 2, int EPI = 0>  // TCB: bytes per element of C
 struct Cfg {
   static constexpr int kBRows = BN / CG;
   static constexpr int kABytes = BM * BK * 2;
   static constexpr int kBBytes = kBRows * BK * 2;
   static constexpr int kStageBytes = kABytes + kBBytes;
-  static constexpr int kStages = (196608 / kStageBytes) < 8 ? (196608 / kStageBytes) : 8;
+  // EPI 5 (SwiGLU backward) gives one stage to its h slots
+  static constexpr int kStages = EPI == 5 ? 5 : ((196608 / kStageBytes) < 8 ? (196608 / kStageBytes) : 8);
   static constexpr int kCols = 2 * BN;  // double-buffered fp32 accumulator
   // Epilogue warps: 8 (two per TMEM lane quarter, each taking half the
   // columns) for bf16 outputs, whose epilogues are latency-bound; 4 for fp32
@@ -361,7 +394,9 @@ struct Cfg {
   // (conflict-free both ways)
   static constexpr int kRowBytes = 32 * TCB;
   static constexpr int kPitch = kRowBytes + 16;
-  static constexpr int kStageBufBytes = 32 * kPitch;
+  // EPI 5: a ring of three 2 KB slots per warp, each the gate and up blocks of
+  // h (in) and of dH (out) for 16 columns of dA, 32 rows x 32 bytes apiece
+  static constexpr int kStageBufBytes = EPI == 5 ? 6144 : 32 * kPitch;
   static constexpr int kStagingBytes = kEpiWarps * kStageBufBytes;
   static constexpr int kSmem = kStages * kStageBytes + kStagingBytes + 1024 /*align*/ + 512 /*barriers*/;
 };
@@ -569,7 +604,8 @@ __device__ __forceinline__ float tanh_approx(float x) {
   asm("tanh.approx.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
 }
-__device__ __forceinline__ float silu_f(float v) { return v * fmaf(0.5f, tanh_approx(0.5f * v), 0.5f); }
+__device__ __forceinline__ float sigmoid_f(float v) { return fmaf(0.5f, tanh_approx(0.5f * v), 0.5f); }
+__device__ __forceinline__ float silu_f(float v) { return v * sigmoid_f(v); }
 
 template <typename T>
 __device__ __forceinline__ void store_row32(T* dst, const float* v, int valid) {
@@ -590,7 +626,7 @@ __device__ __forceinline__ void load_row32(const T* src, float* v) {
   for (int i = 0; i < 32; i += NV) unpack16<T>(*reinterpret_cast<const uint4*>(src + i), v + i);
 }
 
-// EPI: 0 Store, 1 StoreBias, 2 Accum, 3 SwigluFwd, 4 ReluSqFwd (values of moe::Epi).
+// EPI: 0 Store, 1 StoreBias, 2 Accum, 3 SwigluFwd, 4 ReluSqFwd, 5 SwigluBwd (values of moe::Epi).
 // CG: 1 = one CTA per 128 x BN tile; 2 = a cluster of two CTAs per 256 x BN
 // tile (the even CTA issues the MMAs; both stage their halves and drain
 // their own accumulator rows).
@@ -600,7 +636,7 @@ __device__ __forceinline__ void load_row32(const T* src, float* v) {
 template <int BN, bool A_MN, bool B_MN, int GROUP, int EPI, typename TC, int CG, int GATHER = 0>
 __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
     gemm_tc_kernel(const __grid_constant__ Params p) {
-  using C = Cfg<BN, CG, sizeof(TC)>;
+  using C = Cfg<BN, CG, sizeof(TC), EPI>;
   constexpr int EW = C::kEpiWarps;
   constexpr int CSTEP = EW / 4;  // epilogue warps sharing a lane quarter
   constexpr int BMP = BM * CG;
@@ -1043,6 +1079,7 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
     const int64_t ldc_b = p.ldc * (int64_t)sizeof(TC);
     int acc = 0;
     uint32_t acc_phase = 0;
+    int hq = 0;  // EPI 5: ring slot of the current tile's first half
     Walker wk = make_walker<GROUP>(cta0, ncta, total, kper, knce, knz, ktot, ksnake);
     for (int t; next_tile<GROUP>(wk, s_off, s_pref, t);) {
       Tile ti;
@@ -1089,6 +1126,26 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
         for (int i = 0; i < kPre; ++i)
           if (ch + i * CSTEP < nch_acc) acc_fetch(c_rows, ldc_b, n0 + (ch + i * CSTEP) * 32, lane, nrows, pre[i]);
       }
+      // EPI 5: this warp's columns of dA go in halves of 16 (half k of the tile:
+      // chunk k / 2, i.e. columns 32 (ch + CSTEP k / 2) + 16 (k mod 2)) through a
+      // ring of three slots.  The gate and up blocks of h for halves 0 and 1 are
+      // copied in before the accumulator wait; half k + 2's when half k starts,
+      // into the slot that half k - 1 has just written out.  Every half commits
+      // one cp.async group (empty past the tile's last column).
+      const uint8_t* h_rows = EPI == 5 ? static_cast<const uint8_t*>(p.aux) + rbase * ldc_b : nullptr;
+      const uint32_t hs = smem_u32(stg);
+      auto hcol = [&](int k) -> int64_t {  // column of h's gate block for half k
+        const int64_t f = n0 + (ch + (k >> 1) * CSTEP) * 32 + (k & 1) * 16;
+        return (f >> 6) * 128 + (f & 63);
+      };
+      auto hvalid = [&](int k) { return ch + (k >> 1) * CSTEP < nch_acc; };
+      if (EPI == 5) {
+#pragma unroll
+        for (int k = 0; k < 2; ++k) {
+          if (hvalid(k)) h_fetch(hs + ((hq + k) % 3) * 2048, h_rows, ldc_b, hcol(k), lane, nrows);
+          else cp_async_commit();
+        }
+      }
       if (!wait_bounded(smem_u32(&tfull[acc]), acc_phase, &s_abort, p.err)) break;
       tc_fence_after();
       const uint32_t tbase = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
@@ -1131,6 +1188,59 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
             stage_store<RB>(stg, lane, a_rows + (cb / 2 + half * 32) * sizeof(TC), lda_b, nrows);
           }
         }
+      } else if (EPI == 5) {
+        // the SwiGLU backward on the accumulator dA: per 16 columns of dA, the
+        // 16 gate and 16 up columns of h in, the same columns of dH out, each
+        // lane on its own row of the slot
+        constexpr int NH = 2 * (BN / 32 / CSTEP);  // halves per tile
+        uint32_t ra[32];
+#pragma unroll
+        for (int k = 0; k < NH; ++k) {
+          const uint32_t slot = hs + ((hq + k) % 3) * 2048;
+          if (k + 2 < NH && hvalid(k + 2))
+            h_fetch(hs + ((hq + k + 2) % 3) * 2048, h_rows, ldc_b, hcol(k + 2), lane, nrows);
+          else
+            cp_async_commit();
+          cp_async_wait_group<2>();  // half k's group: only halves k + 1 and k + 2 may still be in flight
+          __syncwarp();
+          if (hvalid(k)) {
+            const int c = ch + (k >> 1) * CSTEP;
+            if ((k & 1) == 0) tmem_ld32_issue(tbase + c * 32, ra);
+            float g[16], u[16];
+#pragma unroll
+            for (int j = 0; j < 2; ++j) {
+              unpack16<TC>(lds128(slot + hs_off(lane, j)), g + j * Vec<TC>::N);
+              unpack16<TC>(lds128(slot + 1024 + hs_off(lane, j)), u + j * Vec<TC>::N);
+            }
+            if ((k & 1) == 0) tmem_ld_wait(ra);
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {
+              const float a = __uint_as_float(ra[(k & 1) * 16 + j]);
+              const float s = sigmoid_f(g[j]);
+              const float dg = a * u[j] * s * (1.0f + g[j] * (1.0f - s));
+              u[j] = a * g[j] * s;
+              g[j] = dg;
+            }
+#pragma unroll
+            for (int j = 0; j < 2; ++j) {
+              sts128(slot + hs_off(lane, j), pack16<TC>(g + j * Vec<TC>::N));
+              sts128(slot + 1024 + hs_off(lane, j), pack16<TC>(u + j * Vec<TC>::N));
+            }
+            __syncwarp();
+            const int64_t gc = hcol(k);
+#pragma unroll
+            for (int it = 0; it < 2; ++it) {
+              const int r = it * 16 + lane / 2, pc = lane % 2;
+              if (r < nrows) {
+                uint8_t* dst = c_rows + r * ldc_b + gc * 2 + pc * 16;
+                *reinterpret_cast<uint4*>(dst) = lds128(slot + hs_off(r, pc));
+                *reinterpret_cast<uint4*>(dst + 128) = lds128(slot + 1024 + hs_off(r, pc));
+              }
+            }
+            __syncwarp();  // the slot is read out before it is refilled
+          }
+        }
+        hq = (hq + NH) % 3;
       } else if (EPI == 2) {
         // C += acc, with the C blocks fetched above
 #pragma unroll
@@ -1245,6 +1355,7 @@ __global__ void __launch_bounds__(Cfg<BN, CG, sizeof(TC)>::kThreads, 1)
       }
       if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
     }
+    if (EPI == 5) cp_async_wait_all();  // no h copy is still landing when the CTA exits
   }
 
   tc_fence_before();

@@ -135,6 +135,8 @@ enum class Epi : int {
   Accum = 2,      // C = C + acc
   SwigluFwd = 3,  // acc is h (packed gate/up, N = 2F): C = h, aux[m, f] = silu(g) u  (aux ld = N/2)
   ReluSqFwd = 4,  // acc is h: C = h, aux[m, n] = max(h, 0)^2  (aux ld = ldc)
+  SwigluBwd = 5,  // acc is dA (N = F); aux is the saved h (packed gate/up blocks of 64, ld = ldc = 2N):
+                  // C = dH in h's layout, dg = dA u s (1 + g (1 - s)), du = dA g s, s = sigmoid(g)
 };
 
 struct GemmDesc {
@@ -154,7 +156,8 @@ struct GemmDesc {
   DType c_type = DType::BF16;
   int64_t ldc = 0, sc_g = 0;
   const float* bias = nullptr;       // StoreBias
-  void* aux = nullptr;               // SwigluFwd / ReluSqFwd activation output (c_type)
+  void* aux = nullptr;               // SwigluFwd / ReluSqFwd activation output (c_type);
+                                     // SwigluBwd: the saved h, only read
   void* scratch = nullptr;           // Group::K on the tensor-core engine: per-group tensor maps
                                      // (gemm_tc_group_scratch_bytes, 128-byte aligned)
   bool maps_ready = false;           // Group::K: the maps in scratch were already built
