@@ -225,9 +225,9 @@ int moe_combine_bwd(const moe_shape_t* shape, const void* dy, const void* y_perm
  * dx_perm = dH . w1_e, dw2_e = dy_perm_e^T . a_e, dw1_e = dH_e^T . x_perm_e.
  * dw1 [E, 2F, D] and dw2 [E, D, F] are fp32 and fully written (zero for an
  * expert with no rows).  dH [TK, 2F] lives in the workspace.  With bf16 operands
- * and F a multiple of 64 the SwiGLU backward runs in dA's GEMM on its fp32
- * accumulator (dA is never stored); otherwise dA is stored in the workspace in
- * the layer's dtype and a separate pass reads it back. */
+ * the SwiGLU backward runs in dA's GEMM on its fp32 accumulator (dA is never
+ * stored); with fp32 operands dA is stored in the workspace and a separate pass
+ * reads it back. */
 int moe_expert_ffn_bwd(const moe_shape_t* shape, const void* dy_perm, const void* x_perm, const void* h_save,
                        const void* act_save, const int32_t* expert_offsets, const void* w1, const void* w2,
                        void* dx_perm, float* dw1, float* dw2, void* ws, size_t ws_bytes, void* stream);
