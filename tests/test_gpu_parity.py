@@ -28,6 +28,10 @@ CASES = {
     "mid_latent": W("mid_latent", S=300, GBS=2, D=256, E=32, K=4, F=192, H=512),
     "mid_fp32": W("mid_fp32", S=300, GBS=1, D=192, E=12, K=3, F=192, dtype="f32"),
     "wide_bf16": W("wide_bf16", S=384, GBS=1, D=1024, E=8, K=2, F=768),
+    # three to four tiles per CTA pair in every grouped GEMM, with a partial last
+    # column tile (F = 320): the epilogues' per-warp state carried from one tile
+    # to the next (the SwiGLU backward's h-slot ring) meets ragged tiles
+    "many_ragged": W("many_ragged", S=8192, GBS=2, D=256, E=8, K=2, F=320),
 }
 
 _cache = {}
