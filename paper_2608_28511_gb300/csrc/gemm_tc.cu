@@ -157,8 +157,9 @@ int max_pair_clusters(KernelT k, int smem, int threads) {
 template <int BN, bool A_MN, bool B_MN, int GROUP, int EPI, typename TC, int CG, int GATHER = 0>
 cudaError_t launch_inst(const Ctx& c, const Params& p, int64_t ub) {
   auto k = tc::gemm_tc_kernel<BN, A_MN, B_MN, GROUP, EPI, TC, CG, GATHER>;
-  constexpr int kSmem = Cfg<BN, CG, sizeof(TC), EPI>::kSmem;
-  constexpr int kThreads = Cfg<BN, CG, sizeof(TC)>::kThreads;
+  constexpr int kZW = (GROUP == 2 && sizeof(TC) == 4 && GATHER == 0) ? 1 : 0;
+  constexpr int kSmem = Cfg<BN, CG, sizeof(TC), EPI, kZW>::kSmem;
+  constexpr int kThreads = Cfg<BN, CG, sizeof(TC), EPI, kZW>::kThreads;
   static bool configured = false;
   static int pairs = 0;
   if (!configured) {
